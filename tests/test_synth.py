@@ -1,0 +1,100 @@
+"""The seeded input generator: Philox4x32-10 known answers, an independent
+Philox implementation, the Irwin-Hall normal and the per-buffer recipes."""
+import numpy as np
+import pytest
+
+import synth
+from conftest import read_golden
+
+
+def test_philox_known_answers():
+    for row in read_golden("philox4x32_10_kat.txt"):
+        v = [int(x, 16) for x in row]
+        assert synth.philox(v[0:4], v[4:6]) == v[6:10]
+
+
+_TRITON_SCRIPT = r"""
+import json, sys
+import numpy as np
+import torch
+import triton
+import triton.language as tl
+
+@triton.jit
+def k(c0, c1, c2, c3, o0, o1, o2, o3, seed, N: tl.constexpr):
+    offs = tl.arange(0, N)
+    r0, r1, r2, r3 = tl.philox(seed, tl.load(c0 + offs), tl.load(c1 + offs), tl.load(c2 + offs),
+                               tl.load(c3 + offs))
+    tl.store(o0 + offs, r0)
+    tl.store(o1 + offs, r1)
+    tl.store(o2 + offs, r2)
+    tl.store(o3 + offs, r3)
+
+ctr = np.array(json.loads(sys.argv[1]), dtype=np.uint32)
+seed = int(sys.argv[2])
+N = ctr.shape[1]
+ins = [torch.from_numpy(ctr[i].view(np.int32).copy()) for i in range(4)]
+outs = [torch.zeros(N, dtype=torch.int32) for _ in range(4)]
+k[(1,)](*ins, *outs, seed, N=N)
+print(json.dumps([[int(x) & 0xFFFFFFFF for x in o.tolist()] for o in outs]))
+"""
+
+
+def test_philox_matches_triton_interpreter():
+    """Triton's tl.philox, run by its CPU interpreter, is an independent
+    Philox4x32-10 implementation."""
+    import json
+    import os
+    import subprocess
+    import sys
+    pytest.importorskip("triton")
+    rng = np.random.default_rng(5)
+    N = 16
+    ctr = rng.integers(0, 2**32, size=(4, N), dtype=np.uint64)
+    seed = int(rng.integers(0, 2**62))
+    env = dict(os.environ, TRITON_INTERPRET="1")
+    r = subprocess.run([sys.executable, "-c", _TRITON_SCRIPT, json.dumps(ctr.tolist()), str(seed)],
+                       capture_output=True, text=True, env=env, timeout=300)
+    if r.returncode != 0:
+        pytest.skip("triton interpreter unavailable: %s" % r.stderr.strip().splitlines()[-1:])
+    outs = json.loads(r.stdout.strip().splitlines()[-1])
+    for j in range(N):
+        ref = synth.philox([int(ctr[i][j]) for i in range(4)], [seed & 0xFFFFFFFF, seed >> 32])
+        assert [outs[i][j] for i in range(4)] == ref
+
+
+def test_irwin_hall_normal_moments():
+    z = np.array([synth.normal_at(synth.P, i) for i in range(200000)])
+    assert abs(z.mean()) < 0.01
+    assert abs(z.std() - 1.0) < 0.01
+    assert np.all(np.abs(z) <= 6.0)
+    # the sum of 12 uniforms has excess kurtosis -1.2/12 = -0.1
+    k = ((z - z.mean()) ** 4).mean() / z.var() ** 2 - 3.0
+    assert -0.15 < k < -0.05
+
+
+def test_buffer_recipes():
+    n = 200000
+    p, m, v = synth.state(n)
+    assert abs(p.std() - 0.02) < 0.0005
+    assert abs(m.std() - 1e-4) < 3e-6
+    assert np.all(v >= 0)
+    assert abs(v.mean() - 1e-6) < 3e-8      # E[x^2] for x ~ N(0, 1e-3)
+    g = synth.grad(n, step=1)
+    gf = (g.astype(np.uint32) << 16).view(np.float32)
+    zero = g == 0
+    assert 0.008 < zero.mean() < 0.012
+    assert abs(gf[~zero].std() - 1e-3) < 3e-5
+    # a later step draws a fresh gradient
+    assert np.mean(synth.grad(n, step=2) == g) < 0.02
+
+
+def test_fill_is_position_pure_and_thread_invariant():
+    n = 300001
+    for kind in (synth.P, synth.M, synth.V, synth.G):
+        a = synth.fill(kind, n, goff=(1 << 32) - 1000, step=3, nthreads=1)
+        b = synth.fill(kind, n, goff=(1 << 32) - 1000, step=3, nthreads=7)
+        assert np.array_equal(a.view(np.uint8), b.view(np.uint8))
+        idx = np.array([(1 << 32) - 1000 + j for j in (0, 1, 999, 1000, 1001, n - 1)], dtype=np.uint64)
+        c = synth.fill_at(kind, idx, step=3)
+        assert np.array_equal(c.view(np.uint8), a[idx - idx[0]].view(np.uint8))
