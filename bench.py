@@ -1,0 +1,411 @@
+#!/usr/bin/env python3
+"""Benchmark of the committed optimizer step with state digest on GB300.
+
+One step = the whole hot path over one rank's shard: ``apc_commit_step``
+(fused AdamW + bf16 copy + four digests) followed by the ``apc_digest``
+verification pass over the written buffers.  Workload (default): the full
+Mistral-7B model on one GPU, 291 separately allocated tensors, 7,248,023,552
+elements (~116 GB of fp32 state), optimizer step 18.  The state is larger
+than L2 (129 MB), so no flush is needed between timed steps.
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
+a bounded sample of the same workload instead.
+
+Multi-GPU (torchrun): every rank runs its own replica of the shard (the
+replication group of hybrid sharding), with no collective on the data path;
+a Gloo control plane brackets the timed region with barriers, takes the
+maximum time over ranks, and checks after timing that all replicas hold
+identical digests.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+M64 = (1 << 64) - 1
+HP = dict(lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1)
+METRIC = "commit-step elements/s and HBM GB/s (fraction of GB300 peak), ms per 7.25B-param step"
+COMMIT_BYTES = 28   # per element: p, m, v fp32 read+write (24) + bf16 g read (2) + bf16 w write (2)
+VERIFY_BYTES = 14   # per element: p, m, v fp32 (12) + bf16 w (2) read
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ----------------------------------------------------------------- helpers
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_18178_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch of ``kernel`` from the committed ncu summary,
+    if it was taken on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[kernel]
+    except (OSError, KeyError, ValueError):
+        return None
+    if rec.get("source_hash") != kernel_source_hash():
+        return None
+    if rec.get("workload") != workload:
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+    FIELDS = ["clocks.sm", "clocks.max.sm", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap", "power.draw"]
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        self.lines = []
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(device_index), "--query-gpu=" + ",".join(self.FIELDS),
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        sm, smax, reasons, power = [], None, set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) != len(self.FIELDS):
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax = float(parts[1])
+                power.append(float(parts[6]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[2:6]):
+                if val.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+# -------------------------------------------------------- distributed setup
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def init_control_plane(world: int):
+    """Gloo process group for barriers and the post-step digest exchange."""
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+    dist.init_process_group("gloo")
+    return dist
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def max_over_ranks(dist, x: float) -> float:
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replicas_agree(dist, digests: list[int]) -> bool:
+    """All ranks hold identical digests (the replica check of recovery)."""
+    if dist is None:
+        return True
+    gathered = [None] * dist.get_world_size()
+    dist.all_gather_object(gathered, [int(d) & M64 for d in digests])
+    return all(g == gathered[0] for g in gathered)
+
+
+# ------------------------------------------------------------- GPU arm
+
+def run_gpu(args):
+    import torch
+    import paper_2609_18178_gb300 as apc
+    import synth
+    from synth import workloads as W
+
+    world, rank, local = dist_env()
+    dist = init_control_plane(world)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = W.ALL[args.workload]()
+    step_t = w.steps[-1]
+    N = w.n
+
+    # resident state: one allocation per tensor, filled by the device generator
+    stream = torch.cuda.current_stream()
+    s = stream.cuda_stream
+    bufs = []
+    goff_of = {}
+    for pc in w.pieces:
+        goff_of.setdefault(pc.alloc, pc.goff - pc.at)
+    for a, n in enumerate(w.allocs):
+        b = dict(p=torch.empty(n, dtype=torch.float32, device=dev), m=torch.empty(n, dtype=torch.float32, device=dev),
+                 v=torch.empty(n, dtype=torch.float32, device=dev), g=torch.empty(n, dtype=torch.int16, device=dev),
+                 w=torch.empty(n, dtype=torch.int16, device=dev))
+        g0 = goff_of[a]
+        synth.fill_dev(synth.P, b["p"].data_ptr(), n, g0, stream=s)
+        synth.fill_dev(synth.M, b["m"].data_ptr(), n, g0, stream=s)
+        synth.fill_dev(synth.V, b["v"].data_ptr(), n, g0, stream=s)
+        synth.fill_dev(synth.G, b["g"].data_ptr(), n, g0, step=step_t, stream=s)
+        bufs.append(b)
+    entries, vbufs = [], []
+    for pc in w.pieces:
+        b = bufs[pc.alloc]
+        sl = slice(pc.at, pc.at + pc.n)
+        entries.append(apc.TensorEntry(b["p"][sl], b["m"][sl], b["v"][sl], b["g"][sl], b["w"][sl], pc.goff))
+        vbufs += apc.state_buffers(b["p"][sl], b["m"][sl], b["v"][sl], b["w"][sl], pc.goff)
+    out_c = torch.empty(4, dtype=torch.int64, device=dev)
+    out_v = torch.empty(4, dtype=torch.int64, device=dev)
+    torch.cuda.synchronize()
+
+    def one_step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        apc.commit_step(entries, step_t, HP, stream=s, out=out_c)
+        if ev is not None:
+            ev[1].record(stream)
+        apc.digest(vbufs, 4, stream=s, out=out_v)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    clocks = ClockSampler(local) if not args.no_clocks else None
+    barrier(dist)
+    torch.cuda.synchronize()
+    for k in range(K):
+        one_step(evs[k])
+    torch.cuda.synchronize()
+    barrier(dist)
+    clk = clocks.stop() if clocks else None
+    commit_ms = [evs[k][0].elapsed_time(evs[k][1]) for k in range(K)]
+    verify_ms = [evs[k][1].elapsed_time(evs[k][2]) for k in range(K)]
+    total_ms = evs[0][0].elapsed_time(evs[K - 1][2])
+    total_ms = max_over_ranks(dist, total_ms)
+    ms_per_step = total_ms / K
+    digests_c = apc.digests_to_host(out_c)
+    digests_v = apc.digests_to_host(out_v)
+    agree = replicas_agree(dist, digests_c + digests_v)
+
+    # end to end: the step's gradient from pinned host memory, the digests back
+    e2e = None
+    if not args.no_e2e:
+        host_g = []
+        for b in bufs:
+            hg = torch.empty(b["g"].numel(), dtype=torch.int16, pin_memory=True)
+            hg.copy_(b["g"])
+            host_g.append(hg)
+        host_out = torch.empty(8, dtype=torch.int64, pin_memory=True)
+        torch.cuda.synchronize()
+
+        def e2e_step():
+            for b, hg in zip(bufs, host_g):
+                b["g"].copy_(hg, non_blocking=True)
+            one_step()
+            host_out[:4].copy_(out_c, non_blocking=True)
+            host_out[4:].copy_(out_v, non_blocking=True)
+
+        for _ in range(max(1, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize()
+        ke = max(1, min(K, args.e2e_steps))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(dist)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(ke):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(dist)
+        e2e_ms = max_over_ranks(dist, e0.elapsed_time(e1)) / ke
+        e2e = {"value": world * N / (e2e_ms * 1e-3), "unit": "elements/s",
+               "h2d_bytes_per_step": 2 * N, "d2h_bytes_per_step": 64, "ms_per_step": e2e_ms, "steps": ke}
+        del host_g
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, step_t, args.cpu_seconds)
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+    peak, peak_kind = measured_peak()
+    c_ms = statistics.median(commit_ms)
+    v_ms = statistics.median(verify_ms)
+    c_avg = sum(commit_ms) / K
+    achieved = COMMIT_BYTES * N / (c_avg * 1e-3) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": world * N / (ms_per_step * 1e-3),
+        "unit": "elements/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32+u64",
+        "data": "synthetic",
+        "config": {"workload": "%s: full Mistral-7B shard on one GPU, %d tensors, %d elements, step %d, "
+                               "commit+digest then re-verify" % (w.name, len(w.pieces), N, step_t),
+                   "elements": N, "tensors": len(w.pieces), "step": step_t, "parallelism": "replica x%d" % world,
+                   "l2": "inputs larger than L2 (%.0f GB resident state)" % (16 * N / 1e9)},
+        "hbm_gbs_step": (COMMIT_BYTES + VERIFY_BYTES) * N / (ms_per_step * 1e-3) / 1e9,
+        "commit_ms": c_ms,
+        "verify_ms": v_ms,
+        "commit_gbs": COMMIT_BYTES * N / (c_ms * 1e-3) / 1e9,
+        "verify_gbs": VERIFY_BYTES * N / (v_ms * 1e-3) / 1e9,
+        "commit_elements_per_s": N / (c_ms * 1e-3),
+        "frac_of_spec_8tbs": achieved / 8000.0,
+        "roofline": {"bound": "hbm", "kernel": "commit_kernel", "achieved": achieved, "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": profiled_traffic("commit_kernel", w.name),
+                     "algorithmic_bytes_per_launch": COMMIT_BYTES * N},
+        "gpu_launches": K * (1 + (len(vbufs) + 999) // 1000),
+        "digests": ["%016x" % d for d in digests_c],
+        "verify_matches_commit": digests_c == digests_v,
+        "replica_digests_agree": agree,
+        "clocks": clk,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+# --------------------------------------------------------- CPU oracle arm
+
+def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
+    """The oracle (as it stands) on all host cores over a bounded sample: the
+    first ``sample`` elements of the workload's flat order, repeated until
+    ``seconds`` of work; input generation is not timed."""
+    import oracle
+    import synth
+    n = min(sample, w.n)
+    cores = os.cpu_count() or 1
+    g0 = w.pieces[0].goff
+    p, m, v = synth.state(n, g0)
+    g = synth.grad(n, g0, step_t)
+    h8 = oracle.resolve_hparams(HP, step_t)
+    done, t0 = 0, time.perf_counter()
+    while True:
+        oracle.commit(p, m, v, g, g0, h8, nthreads=cores)
+        done += n
+        el = time.perf_counter() - t0
+        if el >= seconds or el * (done + n) / done > 3 * seconds:
+            break
+    return {"value": done / el, "unit": "elements/s", "cores": cores, "kind": "oracle",
+            "sample": "first %d elements of %s (embed_tokens), step %d, %d passes, %.1f s" % (n, w.name, step_t,
+                                                                                          done // n, el)}
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from synth import workloads as W
+    w = W.ALL[args.workload]()
+    step_t = w.steps[-1]
+    # each "step" is a bounded sample of the workload on the host cores
+    per_step = max(1.0, args.cpu_seconds / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        cpu_baseline(w, step_t, per_step)
+    vals = [cpu_baseline(w, step_t, per_step) for _ in range(args.steps)]
+    v = statistics.median(x["value"] for x in vals)
+    cb = dict(vals[0], value=v)
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "elements/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * w.n / v, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32+u64", "data": "synthetic",
+            "config": {"workload": "%s (CPU oracle on a bounded sample)" % w.name, "elements": w.n,
+                       "step": step_t},
+            "cpu_baseline": cb,
+            "e2e": {"value": v, "unit": "elements/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=["c1", "c2", "c3", "c4", "c5"], default="c5")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "ours":
+        print("note: at least 3 warm-up steps are required for a valid number", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

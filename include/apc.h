@@ -1,0 +1,161 @@
+/*
+ * apc: the committed optimizer step of zero-I/O fault recovery, as a C ABI.
+ *
+ * arxiv 2609.18178 recovers sharded training in place when a collective
+ * fails at a committed optimizer boundary: the point where the parameter
+ * and moment updates of the step have landed, flat-parameter gradients are
+ * zeroed and device streams are synchronized (Section I; Section III-C,
+ * phase 2).  The device state it keeps is S_app = {W, M, V, ..., tau_opt}
+ * (Section III-A, Eq. 2), and it relies on every rank holding bit-identical
+ * parameter and optimizer state after repair (Abstract; Sections IV-F and
+ * IV-G, "rank state checks passing bitwise").
+ *
+ * This library computes, on one GPU, the step that reaches that boundary for
+ * one rank's flat parameter shard, and a 64-bit digest per state buffer that
+ * lets peers prove bit-identity by exchanging 32 bytes instead of
+ * checkpoints:
+ *
+ *   apc_commit_step  AdamW update of fp32 master params p and moments m, v
+ *                    from a bf16 gradient g, a bf16 copy w of p', and the
+ *                    digests of p', m', v', w, in one pass over HBM.
+ *   apc_digest       the same digests of arbitrary buffers, read-only (the
+ *                    post-recovery verification).
+ *
+ * Numeric contract (identical bits on every run, grid size and table split):
+ *   scalars  b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/(1-b1^t), 1/sqrt(1-b2^t),
+ *            each formed in double from the hyper-parameters and rounded once
+ *            to binary32 on the host (apc_resolve_hparams);
+ *   update   per element, binary32, one rounding per operation, no fusion:
+ *              g  = bf16 -> f32 (exact)
+ *              m' = b1*m + (1-b1)*g
+ *              v' = b2*v + (1-b2)*(g*g)
+ *              den = sqrt(v') * rsb2 + eps          (IEEE sqrt)
+ *              p' = p*(1-lr*wd) - step*(m'/den)     (IEEE divide)
+ *              w  = bf16 round-to-nearest-even of p'
+ *   digest   D_B = sum over elements of
+ *              splitmix64(((G mod 2^32) << 32) | bits_B)   (mod 2^64)
+ *            G the element's index in the flat model (global_offset + i),
+ *            bits_B its binary32 bits or zero-extended bf16 bits, and
+ *            splitmix64(x) the first output of SplitMix64 seeded with x.
+ *            Only G mod 2^32 enters the key: equal words exactly k*2^32
+ *            elements apart have equal keys.
+ *
+ * Conventions for every call:
+ *   - Device pointers belong to the calling thread's current CUDA device.
+ *     The caller owns all memory; the library allocates nothing and keeps
+ *     no state between calls.
+ *   - Work is enqueued on `stream` (NULL = the legacy default stream); the
+ *     call never synchronizes.  Results, including the digests, are valid
+ *     once the stream reaches that point.
+ *   - Tables and buffer lists are read before the call returns; the caller
+ *     may reuse them at once.
+ *   - Errors are returned, never raised: no call aborts the process.  On an
+ *     error before launch nothing is enqueued.  apc_last_error() gives a
+ *     human-readable detail of the calling thread's last failure.
+ */
+#ifndef APC_H
+#define APC_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* The same type as cudaStream_t. */
+typedef struct CUstream_st *apc_stream_t;
+
+typedef enum apc_status {
+  APC_OK = 0,
+  APC_EINVAL = 1, /* null pointer, bad count, out-of-range hyper-parameter or step,
+                     overlapping outputs                                          */
+  APC_EALIGN = 2, /* pointer not aligned to its element size                       */
+  APC_ERANGE = 3, /* global_offset + n overflows 64 bits                           */
+  APC_ECUDA = 4   /* the CUDA runtime reported an error (launch or attribute query) */
+} apc_status;
+
+/* Decimal AdamW hyper-parameters (double).  Valid: lr >= 0, 0 <= beta < 1,
+ * eps > 0, weight_decay >= 0, all finite. */
+typedef struct apc_adamw_hparams {
+  double lr, beta1, beta2, eps, weight_decay;
+} apc_adamw_hparams;
+
+/* One entry of the chunk table: a tensor of the flat shard, or a slice of it.
+ *   p, m, v  fp32, device, n elements each, read and updated in place
+ *   g        bf16 bits, device, n elements, read only
+ *   w        bf16 bits, device, n elements, written (p' rounded to bf16)
+ *   global_offset  index of element 0 in the flat model (the digest key)
+ * p, m, v need 4-byte and g, w 2-byte alignment; the kernel runs 16-byte
+ * vectors wherever the five buffers are mutually aligned and scalar code
+ * elsewhere.  n == 0 entries are skipped and their pointers may be NULL.
+ * The written ranges of all entries (p, m, v, w) must not overlap each other
+ * or any gradient range. */
+typedef struct apc_tensor {
+  float *p, *m, *v;
+  const uint16_t *g;
+  uint16_t *w;
+  uint64_t n;
+  uint64_t global_offset;
+} apc_tensor;
+
+typedef enum apc_dtype { APC_F32 = 0, APC_BF16 = 1 } apc_dtype;
+
+/* One buffer for apc_digest: n elements of `dtype` at `data` (device), whose
+ * element 0 has index global_offset in the flat model, summed into digest
+ * slot `slot`. */
+typedef struct apc_buffer {
+  const void *data;
+  uint64_t n;
+  uint64_t global_offset;
+  uint32_t dtype; /* apc_dtype */
+  uint32_t slot;
+} apc_buffer;
+
+#define APC_MAX_SLOTS 8
+
+/* The committed AdamW step plus state digest over a chunk table.
+ *
+ * table[0..num_tensors): the tensors of one rank's shard (any number; tables
+ *   larger than one launch's capacity are split into several launches on
+ *   `stream`, with identical results).  num_tensors == 0 is valid.
+ * hp, step: hyper-parameters and the 1-based optimizer step t (tau_opt).
+ * out_digests: device, 4 x uint64, written as {D_p', D_m', D_v', D_w}; it is
+ *   zeroed on `stream` first, so it need not be initialised.
+ * Returns APC_EINVAL (null table with num_tensors > 0, null hp or
+ * out_digests, num_tensors < 0, step < 1, hyper-parameters out of range,
+ * overlapping outputs), APC_EALIGN, APC_ERANGE, APC_ECUDA, or APC_OK. */
+apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
+                           int64_t step, apc_stream_t stream, uint64_t *out_digests);
+
+/* The state digest of a list of buffers, read only.
+ *
+ * bufs[0..num_bufs): buffers; each adds its elements into out_digests[slot].
+ * num_slots: 1..APC_MAX_SLOTS; out_digests (device, num_slots x uint64) is
+ *   zeroed on `stream` first.
+ * The digest of the four buffers that apc_commit_step wrote, given as slots
+ * 0..3 with the table's offsets, equals that call's out_digests.
+ * Returns APC_EINVAL (null pointers, bad counts, bad dtype, slot >=
+ * num_slots), APC_EALIGN, APC_ERANGE, APC_ECUDA, or APC_OK. */
+apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, apc_stream_t stream,
+                      uint64_t *out_digests);
+
+/* The eight binary32 scalars that apc_commit_step passes to the device for
+ * step t, in the order b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/(1-b1^t),
+ * 1/sqrt(1-b2^t).  Host only; no CUDA call.  out: host, 8 floats. */
+apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t step, float out[8]);
+
+/* Static description of a status code. */
+const char *apc_status_string(apc_status s);
+
+/* Detail of the calling thread's last failing call ("" if none).  The
+ * pointer stays valid until that thread's next apc_* call. */
+const char *apc_last_error(void);
+
+/* ABI version of this header: 1. */
+int32_t apc_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* APC_H */

@@ -1,0 +1,230 @@
+"""Python binding of libapc (include/apc.h): argument marshalling only.
+
+Every step of the committed update and of the digest runs in the CUDA
+kernels of ``libapc.so``; this module converts torch tensors (or raw device
+pointers) into the C structures, calls the C ABI, and raises on a non-OK
+status.  There is no CPU fallback: importing the binding without a built
+library, or calling it without a CUDA device, raises.
+
+Entry points mirror the C names:
+
+* :func:`commit_step` -> ``apc_commit_step``: fused AdamW update of the fp32
+  master shard and its moments from a bf16 gradient, the bf16 working copy,
+  and the four state digests (p', m', v', w).
+* :func:`digest` -> ``apc_digest``: the same digests of arbitrary buffers,
+  read only (post-recovery verification).
+* :func:`resolve_hparams` -> ``apc_resolve_hparams``: the step's binary32
+  scalars (host only).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Iterable, Sequence
+
+from . import _build
+
+__all__ = ["TensorEntry", "BufferEntry", "ApcError", "commit_step", "digest", "resolve_hparams",
+           "library", "lib_path", "F32", "BF16", "DEFAULT_HPARAMS"]
+
+F32, BF16 = 0, 1
+MASK64 = (1 << 64) - 1
+DEFAULT_HPARAMS = dict(lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1)
+
+
+class _Tensor(ctypes.Structure):
+    _fields_ = [("p", ctypes.c_void_p), ("m", ctypes.c_void_p), ("v", ctypes.c_void_p), ("g", ctypes.c_void_p),
+                ("w", ctypes.c_void_p), ("n", ctypes.c_uint64), ("global_offset", ctypes.c_uint64)]
+
+
+class _Buffer(ctypes.Structure):
+    _fields_ = [("data", ctypes.c_void_p), ("n", ctypes.c_uint64), ("global_offset", ctypes.c_uint64),
+                ("dtype", ctypes.c_uint32), ("slot", ctypes.c_uint32)]
+
+
+class _HParams(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_double), ("beta1", ctypes.c_double), ("beta2", ctypes.c_double),
+                ("eps", ctypes.c_double), ("weight_decay", ctypes.c_double)]
+
+
+class ApcError(RuntimeError):
+    def __init__(self, status: int, detail: str):
+        super().__init__("%s (%s)" % (detail, _lib_status_string(status)))
+        self.status = status
+
+
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def library():
+    """Load libapc.so (building it first if it is missing or stale)."""
+    global _lib
+    if _lib is None:
+        path = _build.build()
+        lib = ctypes.CDLL(path)
+        vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+        lib.apc_commit_step.argtypes = [vp, i32, vp, i64, vp, vp]
+        lib.apc_commit_step.restype = ctypes.c_int
+        lib.apc_digest.argtypes = [vp, i32, i32, vp, vp]
+        lib.apc_digest.restype = ctypes.c_int
+        lib.apc_resolve_hparams.argtypes = [vp, i64, vp]
+        lib.apc_resolve_hparams.restype = ctypes.c_int
+        lib.apc_status_string.argtypes = [ctypes.c_int]
+        lib.apc_status_string.restype = ctypes.c_char_p
+        lib.apc_last_error.argtypes = []
+        lib.apc_last_error.restype = ctypes.c_char_p
+        lib.apc_version.argtypes = []
+        lib.apc_version.restype = ctypes.c_int32
+        _lib = lib
+    return _lib
+
+
+def _lib_status_string(status: int) -> str:
+    return library().apc_status_string(status).decode()
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        raise ApcError(status, library().apc_last_error().decode() or "apc call failed")
+
+
+def _hp(hp: dict | None) -> _HParams:
+    hp = dict(DEFAULT_HPARAMS, **(hp or {}))
+    return _HParams(hp["lr"], hp["beta1"], hp["beta2"], hp["eps"], hp["weight_decay"])
+
+
+def _ptr(x, itemsize: int | None = None) -> int:
+    """Device address of a torch tensor (checked: CUDA, contiguous, element
+    size) or a raw integer pointer."""
+    if x is None:
+        return 0
+    if isinstance(x, int):
+        return x
+    if not x.is_cuda:
+        raise ValueError("tensor is not on a CUDA device")
+    if not x.is_contiguous():
+        raise ValueError("tensor is not contiguous")
+    if itemsize is not None and x.element_size() != itemsize:
+        raise ValueError("expected %d-byte elements, got %s" % (itemsize, x.dtype))
+    return x.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+@dataclass
+class TensorEntry:
+    """One chunk-table entry: fp32 p, m, v (updated in place), bf16 g (read),
+    bf16 w (written), n elements whose first has index ``global_offset`` in
+    the flat model.  Fields are torch tensors or raw device pointers."""
+    p: object
+    m: object
+    v: object
+    g: object
+    w: object
+    global_offset: int = 0
+    n: int | None = None
+
+    def count(self) -> int:
+        if self.n is not None:
+            return int(self.n)
+        return int(self.p.numel())
+
+
+@dataclass
+class BufferEntry:
+    """One digest buffer: ``data`` (torch tensor or pointer) of ``dtype``
+    (F32 or BF16), n elements at ``global_offset``, summed into ``slot``."""
+    data: object
+    slot: int
+    global_offset: int = 0
+    dtype: int | None = None
+    n: int | None = None
+
+
+def _out(out, nslots: int, like):
+    if out is not None:
+        return out
+    import torch
+    dev = like.device if hasattr(like, "device") else torch.device("cuda", torch.cuda.current_device())
+    return torch.empty(nslots, dtype=torch.int64, device=dev)
+
+
+def commit_step(table: Sequence[TensorEntry], step: int, hparams: dict | None = None, stream=None, out=None):
+    """Enqueue the committed AdamW step + digest over ``table`` on ``stream``.
+
+    Returns the device int64[4] tensor that receives {D_p', D_m', D_v', D_w}
+    (bit patterns of the unsigned digests; see :func:`digests_to_host`)."""
+    table = list(table)
+    arr = (_Tensor * max(1, len(table)))()
+    first = None
+    for i, t in enumerate(table):
+        n = t.count()
+        for name, buf, size in (("p", t.p, 4), ("m", t.m, 4), ("v", t.v, 4), ("g", t.g, 2), ("w", t.w, 2)):
+            if not isinstance(buf, int) and buf is not None and buf.numel() < n:
+                raise ValueError("table[%d].%s has %d < %d elements" % (i, name, buf.numel(), n))
+        arr[i] = _Tensor(_ptr(t.p, 4), _ptr(t.m, 4), _ptr(t.v, 4), _ptr(t.g, 2), _ptr(t.w, 2), n,
+                         int(t.global_offset) & MASK64)
+        if first is None and not isinstance(t.p, int):
+            first = t.p
+    out = _out(out, 4, first)
+    hp = _hp(hparams)
+    _check(library().apc_commit_step(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
+                                     ctypes.c_void_p(_stream(stream)), ctypes.c_void_p(_ptr(out, 8))))
+    return out
+
+
+def digest(buffers: Iterable[BufferEntry], num_slots: int = 4, stream=None, out=None):
+    """Enqueue the read-only digest of ``buffers`` into ``num_slots`` slots.
+    Returns the device int64[num_slots] output tensor."""
+    buffers = list(buffers)
+    arr = (_Buffer * max(1, len(buffers)))()
+    first = None
+    for i, b in enumerate(buffers):
+        dt = b.dtype
+        if dt is None:
+            if isinstance(b.data, int):
+                raise ValueError("buffers[%d]: dtype is required for a raw pointer" % i)
+            dt = F32 if b.data.element_size() == 4 else BF16
+        n = b.n if b.n is not None else b.data.numel()
+        arr[i] = _Buffer(_ptr(b.data, 4 if dt == F32 else 2), int(n), int(b.global_offset) & MASK64, dt,
+                         int(b.slot))
+        if first is None and not isinstance(b.data, int):
+            first = b.data
+    out = _out(out, num_slots, first)
+    _check(library().apc_digest(ctypes.addressof(arr), len(buffers), int(num_slots),
+                                ctypes.c_void_p(_stream(stream)), ctypes.c_void_p(_ptr(out, 8))))
+    return out
+
+
+def digests_to_host(out) -> list[int]:
+    """Copy a digest tensor to the host as unsigned 64-bit Python ints."""
+    return [int(x) & MASK64 for x in out.cpu().tolist()]
+
+
+def resolve_hparams(hparams: dict | None, step: int) -> list[float]:
+    """The eight binary32 scalars of step ``step`` (host only)."""
+    hp = _hp(hparams)
+    out = (ctypes.c_float * 8)()
+    _check(library().apc_resolve_hparams(ctypes.addressof(hp), int(step), ctypes.addressof(out)))
+    return list(out)
+
+
+def state_buffers(p, m, v, w, global_offset: int = 0) -> list[BufferEntry]:
+    """The four digest buffers of one tensor in commit_step's slot order."""
+    return [BufferEntry(p, 0, global_offset, F32), BufferEntry(m, 1, global_offset, F32),
+            BufferEntry(v, 2, global_offset, F32), BufferEntry(w, 3, global_offset, BF16)]
+
+
+__all__ += ["digests_to_host", "state_buffers"]

@@ -1,0 +1,75 @@
+"""In-tree build of libapc.so for sm_103a (nvcc, no cmake).
+
+The three translation units compile in parallel; the result lands in
+``paper_2609_18178_gb300/_build/<machine>/libapc.so`` (git-ignored), next to
+the sources, so a GPU host builds its own copy for its own architecture.
+"""
+from __future__ import annotations
+
+import fcntl
+import os
+import platform
+import subprocess
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(HERE)
+CSRC = os.path.join(HERE, "csrc")
+INCLUDE = os.path.join(ROOT, "include")
+BUILD = os.path.join(HERE, "_build", platform.machine())
+LIB = os.path.join(BUILD, "libapc.so")
+
+ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+# exact IEEE binary32: no contraction into FMA, IEEE divide and sqrt, denormals kept
+NUMERIC = ["-fmad=false", "-prec-div=true", "-prec-sqrt=true", "-ftz=false"]
+UNITS = ["apc_commit.cu", "apc_digest.cu", "apc_host.cpp"]
+
+
+def sources() -> list[str]:
+    out = [os.path.join(CSRC, u) for u in UNITS]
+    out += [os.path.join(CSRC, h) for h in ("apc_internal.h", "apc_device.cuh")]
+    out.append(os.path.join(INCLUDE, "apc.h"))
+    return out
+
+
+def stale() -> bool:
+    if not os.path.exists(LIB):
+        return True
+    t = os.path.getmtime(LIB)
+    return any(os.path.getmtime(s) > t for s in sources())
+
+
+def build(force: bool = False, verbose: bool = False) -> str:
+    """Compile libapc.so if missing or older than its sources; return its path."""
+    os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lk:
+        fcntl.flock(lk, fcntl.LOCK_EX)
+        if not force and not stale():
+            return LIB
+        nvcc = os.environ.get("NVCC", "nvcc")
+        common = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-fvisibility=hidden",
+                         "-I", INCLUDE] + NUMERIC
+        if verbose:
+            common += ["-Xptxas", "-v"]
+        procs, objs = [], []
+        for u in UNITS:
+            obj = os.path.join(BUILD, u + ".o")
+            objs.append(obj)
+            procs.append(subprocess.Popen([nvcc, "-c", os.path.join(CSRC, u), "-o", obj] + common,
+                                          stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True))
+        logs = []
+        for u, p in zip(UNITS, procs):
+            out, _ = p.communicate()
+            logs.append(out)
+            if p.returncode != 0:
+                raise RuntimeError("nvcc failed on %s:\n%s" % (u, out))
+        if verbose:
+            print("".join(logs))
+        tmp = LIB + ".tmp%d" % os.getpid()
+        subprocess.run([nvcc] + ARCH + ["-shared", "-o", tmp] + objs, check=True)
+        os.replace(tmp, LIB)
+    return LIB
+
+
+if __name__ == "__main__":
+    import sys
+    print(build(force="--force" in sys.argv, verbose="-v" in sys.argv))

@@ -1,0 +1,131 @@
+// The read-only state digest over a list of buffers (the verification pass
+// after recovery).  Same tiling as the commit kernel: each buffer's 16-byte
+// aligned body is cut into tiles of kDigestTile elements, a persistent grid
+// strides over the launch's tile space, and the scalar head and tail of a
+// buffer go to the CTA that owns its first tile.
+//
+// A thread keeps one running 64-bit sum for the slot of the buffer it is in;
+// all threads of a CTA visit the same tiles, so slot changes are CTA-uniform
+// and the running sum is flushed (warp shuffle reduce, then a shared-memory
+// atomic) only when the CTA moves to a buffer of another slot and at exit.
+#include <cuda_runtime.h>
+
+#include "../../include/apc.h"
+#include "apc_device.cuh"
+#include "apc_internal.h"
+
+namespace apc {
+namespace {
+
+__device__ __forceinline__ void flush(uint64_t &acc, int slot, unsigned long long *s_acc) {
+  uint64_t x = acc;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+  if ((threadIdx.x & 31) == 0 && slot >= 0 && x) atomicAdd(&s_acc[slot], (unsigned long long)x);
+  acc = 0;
+}
+
+__device__ __forceinline__ uint32_t word_at(const DigestEntry &E, uint64_t i) {
+  return E.dtype == 0 ? reinterpret_cast<const uint32_t *>(E.data)[i]
+                      : (uint32_t) reinterpret_cast<const uint16_t *>(E.data)[i];
+}
+
+template <int MAXE>
+__global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
+                                                          unsigned long long *out) {
+  __shared__ unsigned long long s_acc[APC_MAX_SLOTS];
+  if (threadIdx.x < APC_MAX_SLOTS) s_acc[threadIdx.x] = 0;
+  __syncthreads();
+  uint32_t cur = 0;
+  int slot = -1;
+  uint64_t acc = 0;
+  for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
+    while (cur + 1 < plan.count && tile >= plan.e[cur + 1].tile_begin) ++cur;
+    const DigestEntry &E = plan.e[cur];
+    if ((int)E.slot != slot) {
+      flush(acc, slot, s_acc);
+      slot = E.slot;
+    }
+    const uint64_t local = tile - E.tile_begin;
+    const uint64_t head = E.head;
+    const uint64_t vec_end = head + ((E.n - head) & ~(uint64_t)(kVec - 1));
+    const uint64_t base = head + local * kDigestTile;
+    uint64_t t0 = 0, t1 = 0;
+    if (E.dtype == 0) {
+      const uint32_t *d = reinterpret_cast<const uint32_t *>(E.data);
+      uint4 x[kDigestUnroll][2];
+      bool ok[kDigestUnroll];
+#pragma unroll
+      for (int u = 0; u < kDigestUnroll; ++u) {
+        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
+        ok[u] = i < vec_end;
+        if (ok[u]) {
+          x[u][0] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
+          x[u][1] = __ldcs(reinterpret_cast<const uint4 *>(d + i) + 1);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kDigestUnroll; ++u) {
+        if (!ok[u]) continue;
+        const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
+        t0 += digest_term(G + 0, x[u][0].x) + digest_term(G + 1, x[u][0].y);
+        t1 += digest_term(G + 2, x[u][0].z) + digest_term(G + 3, x[u][0].w);
+        t0 += digest_term(G + 4, x[u][1].x) + digest_term(G + 5, x[u][1].y);
+        t1 += digest_term(G + 6, x[u][1].z) + digest_term(G + 7, x[u][1].w);
+      }
+    } else {
+      const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
+      uint4 x[kDigestUnroll];
+      bool ok[kDigestUnroll];
+#pragma unroll
+      for (int u = 0; u < kDigestUnroll; ++u) {
+        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
+        ok[u] = i < vec_end;
+        if (ok[u]) x[u] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
+      }
+#pragma unroll
+      for (int u = 0; u < kDigestUnroll; ++u) {
+        if (!ok[u]) continue;
+        const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
+        t0 += digest_term(G + 0, x[u].x & 0xFFFFu) + digest_term(G + 1, x[u].x >> 16);
+        t1 += digest_term(G + 2, x[u].y & 0xFFFFu) + digest_term(G + 3, x[u].y >> 16);
+        t0 += digest_term(G + 4, x[u].z & 0xFFFFu) + digest_term(G + 5, x[u].z >> 16);
+        t1 += digest_term(G + 6, x[u].w & 0xFFFFu) + digest_term(G + 7, x[u].w >> 16);
+      }
+    }
+    if (local == 0) {
+      const uint32_t t = threadIdx.x;
+      if (t < head) t0 += digest_term(E.key_base + t, word_at(E, t));
+      if (t >= 32 && t - 32 < E.n - vec_end) {
+        const uint64_t i = vec_end + (t - 32);
+        t0 += digest_term(E.key_base + (uint32_t)i, word_at(E, i));
+      }
+    }
+    acc += t0 + t1;
+  }
+  flush(acc, slot, s_acc);
+  __syncthreads();
+  if (threadIdx.x < APC_MAX_SLOTS && s_acc[threadIdx.x]) atomicAdd(&out[threadIdx.x], s_acc[threadIdx.x]);
+}
+
+}  // namespace
+
+int launch_digest_small(const DigestPlan<kDigestSmall> &plan, unsigned grid, void *stream,
+                        unsigned long long *out) {
+  digest_kernel<kDigestSmall><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
+  return (int)cudaGetLastError();
+}
+
+int launch_digest_large(const DigestPlan<kDigestLarge> &plan, unsigned grid, void *stream,
+                        unsigned long long *out) {
+  digest_kernel<kDigestLarge><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
+  return (int)cudaGetLastError();
+}
+
+int digest_blocks_per_sm(bool large, int *out) {
+  cudaError_t e = large ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<kDigestLarge>, kThreads, 0)
+                        : cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<kDigestSmall>, kThreads, 0);
+  return (int)e;
+}
+
+}  // namespace apc

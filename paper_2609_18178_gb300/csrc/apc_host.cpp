@@ -1,0 +1,320 @@
+// Host side of the C ABI declared in include/apc.h: argument validation,
+// resolution of the step's binary32 scalars (in double, rounded once),
+// conversion of the chunk table into launch plans, and the launches.
+//
+// The library allocates nothing.  Each plan travels in the kernel's
+// parameter block; the digests are accumulated with atomics straight into
+// the caller's output, which is zeroed on the stream first.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <memory>
+#include <mutex>
+#include <vector>
+
+#include "../../include/apc.h"
+#include "apc_internal.h"
+
+#define APC_EXPORT extern "C" __attribute__((visibility("default")))
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+apc_status fail(apc_status s, const char *fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+apc_status cuda_fail(int err, const char *what) {
+  return fail(APC_ECUDA, "%s: %s", what, cudaGetErrorString((cudaError_t)err));
+}
+
+// Scalars of step t (see apc_resolve_hparams).
+apc_status resolve(const apc_adamw_hparams *hp, int64_t step, float out[8]) {
+  if (!hp) return fail(APC_EINVAL, "hparams pointer is null");
+  if (step < 1) return fail(APC_EINVAL, "step %lld < 1", (long long)step);
+  const double lr = hp->lr, b1 = hp->beta1, b2 = hp->beta2, eps = hp->eps, wd = hp->weight_decay;
+  if (!std::isfinite(lr) || !std::isfinite(b1) || !std::isfinite(b2) || !std::isfinite(eps) || !std::isfinite(wd))
+    return fail(APC_EINVAL, "non-finite hyper-parameter");
+  if (!(b1 >= 0.0 && b1 < 1.0) || !(b2 >= 0.0 && b2 < 1.0)) return fail(APC_EINVAL, "beta outside [0, 1)");
+  if (!(eps > 0.0)) return fail(APC_EINVAL, "eps must be > 0");
+  if (lr < 0.0 || wd < 0.0) return fail(APC_EINVAL, "lr and weight_decay must be >= 0");
+  // bias corrections in double; each scalar rounded once to binary32
+  const double bc1 = 1.0 - std::pow(b1, (double)step);
+  const double bc2 = 1.0 - std::pow(b2, (double)step);
+  out[0] = (float)b1;
+  out[1] = (float)(1.0 - b1);
+  out[2] = (float)b2;
+  out[3] = (float)(1.0 - b2);
+  out[4] = (float)eps;
+  out[5] = (float)(1.0 - lr * wd);
+  out[6] = (float)(lr / bc1);
+  out[7] = (float)(1.0 / std::sqrt(bc2));
+  return APC_OK;
+}
+
+struct Range {
+  uintptr_t lo, hi;  // [lo, hi)
+  bool written;
+};
+
+// Written ranges must be pairwise disjoint and disjoint from read ranges.
+bool overlaps(std::vector<Range> &r) {
+  std::sort(r.begin(), r.end(), [](const Range &a, const Range &b) { return a.lo < b.lo; });
+  uintptr_t hi_any = 0, hi_written = 0;
+  bool have_any = false, have_written = false;
+  for (const Range &x : r) {
+    if (have_written && x.lo < hi_written) return true;
+    if (x.written && have_any && x.lo < hi_any) return true;
+    if (!have_any || x.hi > hi_any) hi_any = x.hi;
+    have_any = true;
+    if (x.written) {
+      if (!have_written || x.hi > hi_written) hi_written = x.hi;
+      have_written = true;
+    }
+  }
+  return false;
+}
+
+struct Device {
+  int sms = 0;
+  int commit_small = 0, commit_large = 0, digest_small = 0, digest_large = 0;
+};
+
+constexpr int kMaxDevices = 64;
+Device g_devices[kMaxDevices];
+std::atomic<bool> g_device_ready[kMaxDevices];
+std::mutex g_device_mu;
+
+// SM count and occupancy of the current device, queried once per device.
+apc_status device_info(Device *out) {
+  int dev = 0;
+  int e = (int)cudaGetDevice(&dev);
+  if (e) return cuda_fail(e, "cudaGetDevice");
+  if (dev >= 0 && dev < kMaxDevices && g_device_ready[dev].load(std::memory_order_acquire)) {
+    *out = g_devices[dev];
+    return APC_OK;
+  }
+  Device dd, *d = &dd;
+  e = (int)cudaDeviceGetAttribute(&d->sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e) return cuda_fail(e, "cudaDeviceGetAttribute");
+  if ((e = apc::commit_blocks_per_sm(false, &d->commit_small))) return cuda_fail(e, "occupancy query");
+  if ((e = apc::commit_blocks_per_sm(true, &d->commit_large))) return cuda_fail(e, "occupancy query");
+  if ((e = apc::digest_blocks_per_sm(false, &d->digest_small))) return cuda_fail(e, "occupancy query");
+  if ((e = apc::digest_blocks_per_sm(true, &d->digest_large))) return cuda_fail(e, "occupancy query");
+  if (dev >= 0 && dev < kMaxDevices) {
+    std::lock_guard<std::mutex> lock(g_device_mu);
+    if (!g_device_ready[dev].load(std::memory_order_relaxed)) {
+      g_devices[dev] = dd;
+      g_device_ready[dev].store(true, std::memory_order_release);
+    }
+  }
+  *out = dd;
+  return APC_OK;
+}
+
+unsigned grid_for(uint64_t tiles, int sms, int per_sm) {
+  uint64_t cap = (uint64_t)sms * (uint64_t)std::max(per_sm, 1);
+  return (unsigned)std::max<uint64_t>(1, std::min(tiles, cap));
+}
+
+template <int MAXE, typename Launch>
+apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, const float h[8], unsigned grid_cap,
+                              void *stream, unsigned long long *out, Launch launch) {
+  auto plan = std::make_unique<apc::CommitPlan<MAXE>>();
+  std::memcpy(plan->h, h, sizeof plan->h);
+  size_t i = 0;
+  while (i < entries.size()) {
+    const size_t k = std::min(entries.size() - i, (size_t)MAXE);
+    uint64_t tiles = 0;
+    for (size_t j = 0; j < k; ++j) {
+      apc::CommitEntry e = entries[i + j];
+      const uint64_t t = e.tile_begin;  // holds the entry's tile count until placed
+      e.tile_begin = tiles;
+      tiles += t;
+      plan->e[j] = e;
+    }
+    plan->count = (uint32_t)k;
+    plan->total_tiles = tiles;
+    const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(tiles, grid_cap));
+    int e = launch(*plan, grid, stream, out);
+    if (e) return cuda_fail(e, "commit kernel launch");
+    i += k;
+  }
+  return APC_OK;
+}
+
+template <int MAXE, typename Launch>
+apc_status run_digest_batches(const std::vector<apc::DigestEntry> &entries, unsigned grid_cap, void *stream,
+                              unsigned long long *out, Launch launch) {
+  auto plan = std::make_unique<apc::DigestPlan<MAXE>>();
+  size_t i = 0;
+  while (i < entries.size()) {
+    const size_t k = std::min(entries.size() - i, (size_t)MAXE);
+    uint64_t tiles = 0;
+    for (size_t j = 0; j < k; ++j) {
+      apc::DigestEntry e = entries[i + j];
+      const uint64_t t = e.tile_begin;
+      e.tile_begin = tiles;
+      tiles += t;
+      plan->e[j] = e;
+    }
+    plan->count = (uint32_t)k;
+    plan->total_tiles = tiles;
+    const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(tiles, grid_cap));
+    int e = launch(*plan, grid, stream, out);
+    if (e) return cuda_fail(e, "digest kernel launch");
+    i += k;
+  }
+  return APC_OK;
+}
+
+uint64_t ceil_div(uint64_t a, uint64_t b) { return a / b + (a % b != 0); }
+
+}  // namespace
+
+APC_EXPORT apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t step, float out[8]) {
+  g_last_error[0] = 0;
+  if (!out) return fail(APC_EINVAL, "output pointer is null");
+  return resolve(hp, step, out);
+}
+
+APC_EXPORT apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
+                                      int64_t step, apc_stream_t stream, uint64_t *out_digests) {
+  g_last_error[0] = 0;
+  if (num_tensors < 0) return fail(APC_EINVAL, "num_tensors %d < 0", num_tensors);
+  if (num_tensors > 0 && !table) return fail(APC_EINVAL, "table pointer is null");
+  if (!out_digests) return fail(APC_EINVAL, "out_digests pointer is null");
+  if ((uintptr_t)out_digests % 8) return fail(APC_EALIGN, "out_digests not 8-byte aligned");
+  float h[8];
+  apc_status st = resolve(hp, step, h);
+  if (st != APC_OK) return st;
+
+  std::vector<apc::CommitEntry> entries;
+  std::vector<Range> ranges;
+  entries.reserve((size_t)num_tensors);
+  ranges.reserve((size_t)num_tensors * 5);
+  for (int32_t k = 0; k < num_tensors; ++k) {
+    const apc_tensor &t = table[k];
+    if (t.n == 0) continue;
+    if (!t.p || !t.m || !t.v || !t.g || !t.w) return fail(APC_EINVAL, "table[%d]: null buffer pointer", k);
+    if (t.n > (UINT64_MAX - t.global_offset)) return fail(APC_ERANGE, "table[%d]: global_offset + n overflows", k);
+    if (t.n > ((uint64_t)1 << 61)) return fail(APC_ERANGE, "table[%d]: n too large", k);
+    const uintptr_t p = (uintptr_t)t.p, m = (uintptr_t)t.m, v = (uintptr_t)t.v, g = (uintptr_t)t.g,
+                    w = (uintptr_t)t.w;
+    if (p % 4 || m % 4 || v % 4) return fail(APC_EALIGN, "table[%d]: fp32 buffer not 4-byte aligned", k);
+    if (g % 2 || w % 2) return fail(APC_EALIGN, "table[%d]: bf16 buffer not 2-byte aligned", k);
+    ranges.push_back({p, p + 4 * t.n, true});
+    ranges.push_back({m, m + 4 * t.n, true});
+    ranges.push_back({v, v + 4 * t.n, true});
+    ranges.push_back({w, w + 2 * t.n, true});
+    ranges.push_back({g, g + 2 * t.n, false});
+    // first element at which all five buffers sit on a 16-byte boundary
+    const uint64_t h0 = ((16 - g % 16) % 16) / 2;
+    const bool aligned = (p + 4 * h0) % 16 == 0 && (m + 4 * h0) % 16 == 0 && (v + 4 * h0) % 16 == 0 &&
+                         (w + 2 * h0) % 16 == 0;
+    apc::CommitEntry e;
+    e.p = t.p;
+    e.m = t.m;
+    e.v = t.v;
+    e.g = t.g;
+    e.w = t.w;
+    e.n = t.n;
+    e.key_base = (uint32_t)t.global_offset;
+    if (aligned) {
+      const uint64_t head = std::min<uint64_t>(h0, t.n);
+      const uint64_t body = (t.n - head) / apc::kVec * apc::kVec;
+      e.head = (uint32_t)head;
+      e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kCommitTile));
+    } else {
+      e.head = apc::kScalarMode;
+      e.tile_begin = ceil_div(t.n, apc::kCommitTile);
+    }
+    entries.push_back(e);
+  }
+  if (overlaps(ranges)) return fail(APC_EINVAL, "table buffers overlap (a written range meets another range)");
+
+  int e = (int)cudaMemsetAsync(out_digests, 0, 4 * sizeof(uint64_t), (cudaStream_t)stream);
+  if (e) return cuda_fail(e, "cudaMemsetAsync(out_digests)");
+  if (entries.empty()) return APC_OK;
+  Device d;
+  if ((st = device_info(&d)) != APC_OK) return st;
+  unsigned long long *out = reinterpret_cast<unsigned long long *>(out_digests);
+  if (entries.size() <= (size_t)apc::kCommitSmall)
+    return run_commit_batches<apc::kCommitSmall>(entries, h, grid_for(UINT64_MAX, d.sms, d.commit_small), stream,
+                                                 out, apc::launch_commit_small);
+  return run_commit_batches<apc::kCommitLarge>(entries, h, grid_for(UINT64_MAX, d.sms, d.commit_large), stream,
+                                               out, apc::launch_commit_large);
+}
+
+APC_EXPORT apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, apc_stream_t stream,
+                                 uint64_t *out_digests) {
+  g_last_error[0] = 0;
+  if (num_bufs < 0) return fail(APC_EINVAL, "num_bufs %d < 0", num_bufs);
+  if (num_bufs > 0 && !bufs) return fail(APC_EINVAL, "bufs pointer is null");
+  if (num_slots < 1 || num_slots > APC_MAX_SLOTS)
+    return fail(APC_EINVAL, "num_slots %d outside 1..%d", num_slots, APC_MAX_SLOTS);
+  if (!out_digests) return fail(APC_EINVAL, "out_digests pointer is null");
+  if ((uintptr_t)out_digests % 8) return fail(APC_EALIGN, "out_digests not 8-byte aligned");
+  std::vector<apc::DigestEntry> entries;
+  entries.reserve((size_t)num_bufs);
+  for (int32_t k = 0; k < num_bufs; ++k) {
+    const apc_buffer &b = bufs[k];
+    if (b.dtype != APC_F32 && b.dtype != APC_BF16) return fail(APC_EINVAL, "bufs[%d]: unknown dtype %u", k, b.dtype);
+    if (b.slot >= (uint32_t)num_slots) return fail(APC_EINVAL, "bufs[%d]: slot %u >= num_slots", k, b.slot);
+    if (b.n == 0) continue;
+    if (!b.data) return fail(APC_EINVAL, "bufs[%d]: null data pointer", k);
+    if (b.n > (UINT64_MAX - b.global_offset)) return fail(APC_ERANGE, "bufs[%d]: global_offset + n overflows", k);
+    if (b.n > ((uint64_t)1 << 61)) return fail(APC_ERANGE, "bufs[%d]: n too large", k);
+    const uintptr_t a = (uintptr_t)b.data;
+    const uint64_t es = b.dtype == APC_F32 ? 4 : 2;
+    if (a % es) return fail(APC_EALIGN, "bufs[%d]: data not %u-byte aligned", k, (unsigned)es);
+    apc::DigestEntry e;
+    e.data = b.data;
+    e.n = b.n;
+    e.key_base = (uint32_t)b.global_offset;
+    e.head = (uint8_t)std::min<uint64_t>(((16 - a % 16) % 16) / es, b.n);
+    e.dtype = (uint8_t)b.dtype;
+    e.slot = (uint8_t)b.slot;
+    e.pad_ = 0;
+    const uint64_t body = (b.n - e.head) / apc::kVec * apc::kVec;
+    e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kDigestTile));
+    entries.push_back(e);
+  }
+  int e = (int)cudaMemsetAsync(out_digests, 0, (size_t)num_slots * sizeof(uint64_t), (cudaStream_t)stream);
+  if (e) return cuda_fail(e, "cudaMemsetAsync(out_digests)");
+  if (entries.empty()) return APC_OK;
+  Device d;
+  apc_status st = device_info(&d);
+  if (st != APC_OK) return st;
+  unsigned long long *out = reinterpret_cast<unsigned long long *>(out_digests);
+  if (entries.size() <= (size_t)apc::kDigestSmall)
+    return run_digest_batches<apc::kDigestSmall>(entries, grid_for(UINT64_MAX, d.sms, d.digest_small), stream, out,
+                                                 apc::launch_digest_small);
+  return run_digest_batches<apc::kDigestLarge>(entries, grid_for(UINT64_MAX, d.sms, d.digest_large), stream, out,
+                                               apc::launch_digest_large);
+}
+
+APC_EXPORT const char *apc_status_string(apc_status s) {
+  switch (s) {
+    case APC_OK: return "APC_OK: success";
+    case APC_EINVAL: return "APC_EINVAL: invalid argument";
+    case APC_EALIGN: return "APC_EALIGN: misaligned pointer";
+    case APC_ERANGE: return "APC_ERANGE: index range overflow";
+    case APC_ECUDA: return "APC_ECUDA: CUDA runtime error";
+  }
+  return "unknown apc_status";
+}
+
+APC_EXPORT const char *apc_last_error(void) { return g_last_error; }
+
+APC_EXPORT int32_t apc_version(void) { return 1; }

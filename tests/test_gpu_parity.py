@@ -1,0 +1,344 @@
+"""GPU parity of the CUDA path (through the C ABI) against the CPU oracle.
+
+Bar: every written float and bf16 word bit-identical (0 ulp) and every digest
+equal.  Small cases compare every element; the paper-sized workloads compare
+full digests against the streamed oracle where the host can regenerate them
+in seconds, and sampled elements plus digest properties at the largest size,
+in the same launch configuration the benchmark times.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from synth import workloads as W
+
+from apc_testlib import (M64, DeviceWorkload, gf32, oracle_at, oracle_workload_digest, sample_indices)
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # the CUDA path has no fallback: without a GPU these tests cannot run
+    pytest.skip("no CUDA device", allow_module_level=True)
+
+import paper_2609_18178_gb300 as apc  # noqa: E402
+
+HP = oracle.DEFAULT_HP
+
+
+def dev(a):
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if t.dtype == torch.uint16:
+        t = t.view(torch.int16)
+    return t.cuda()
+
+
+def host(t, dt):
+    return t.cpu().numpy().view(dt)
+
+
+def run_small(tensors, step, hp=HP):
+    """tensors: list of dict(p, m, v, g numpy, goff).  Runs the CUDA path and
+    the oracle on copies; returns (device results, oracle results)."""
+    entries, devs = [], []
+    for t in tensors:
+        d = dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=dev(t["g"]),
+                 w=torch.zeros(t["p"].size, dtype=torch.int16, device="cuda"))
+        devs.append(d)
+        entries.append(apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], t["goff"]))
+    out = apc.commit_step(entries, step, hp)
+    torch.cuda.synchronize()
+    h8 = oracle.resolve_hparams(hp, step)
+    ref = [dict(p=t["p"].copy(), m=t["m"].copy(), v=t["v"].copy(), g=t["g"], goff=t["goff"]) for t in tensors]
+    ws, dref = oracle.commit_table(ref, h8)
+    for r, wv in zip(ref, ws):
+        r["w"] = wv
+    return devs, apc.digests_to_host(out), ref, dref
+
+
+def assert_same(devs, dgot, ref, dref):
+    for d, r in zip(devs, ref):
+        for k in "pmv":
+            a, b = host(d[k], np.uint32), r[k].view(np.uint32)
+            bad = np.nonzero(a != b)[0]
+            assert bad.size == 0, "%s differs at %s: %s vs %s" % (k, bad[:5], a[bad[:5]], b[bad[:5]])
+        a, b = host(d["w"], np.uint16), r["w"]
+        assert np.array_equal(a, b), "w differs"
+    assert dgot == dref, "digests differ"
+
+
+def gen(n, goff, step, seed_shift=0):
+    p, m, v = synth.state(n, goff)
+    return dict(p=p, m=m, v=v, g=synth.grad(n, goff, step), goff=goff)
+
+
+def test_c1_chained_three_steps():
+    w = W.c1()
+    n = w.n
+    t = gen(n, 0, 1)
+    state = dict(p=t["p"], m=t["m"], v=t["v"])
+    d = dict(p=dev(state["p"]), m=dev(state["m"]), v=dev(state["v"]),
+             w=torch.zeros(n, dtype=torch.int16, device="cuda"))
+    for step in (1, 2, 3):
+        g = synth.grad(n, 0, step)
+        d["g"] = dev(g)
+        out = apc.commit_step([apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], 0)], step, HP)
+        torch.cuda.synchronize()
+        wv, dref = oracle.commit(state["p"], state["m"], state["v"], g, 0, oracle.resolve_hparams(HP, step))
+        for k in "pmv":
+            assert np.array_equal(host(d[k], np.uint32), state[k].view(np.uint32)), (step, k)
+        assert np.array_equal(host(d["w"], np.uint16), wv)
+        assert apc.digests_to_host(out) == dref
+        ver = apc.digest(apc.state_buffers(d["p"], d["m"], d["v"], d["w"], 0), 4)
+        assert apc.digests_to_host(ver) == dref
+
+
+@pytest.mark.parametrize("n", list(range(1, 65)) + [127, 129, 4095, 4096, 4097, 8191, 8199, 100003])
+def test_small_sizes(n):
+    goff = (1 << 32) - n // 2 - 3
+    assert_same(*run_small([gen(n, goff, 2)], 2))
+
+
+@pytest.mark.parametrize("goff", [0, 5, (1 << 32) - 1, (1 << 32) + 77, M64 - 70000, (1 << 40) + 3])
+def test_global_offsets(goff):
+    n = 60000 if goff < M64 - 70000 else 70000
+    t = gen(n, 0, 3)
+    t["goff"] = goff
+    assert_same(*run_small([t], 3))
+
+
+@pytest.mark.parametrize("shift", range(1, 8))
+def test_uniform_misalignment_uses_head(shift):
+    """All five buffers start `shift` elements past a 16-byte boundary."""
+    n = 20000 + shift
+    t = gen(n + shift, 100, 4)
+    base = dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=dev(t["g"]),
+                w=torch.zeros(n + shift, dtype=torch.int16, device="cuda"))
+    sl = slice(shift, shift + n)
+    out = apc.commit_step([apc.TensorEntry(base["p"][sl], base["m"][sl], base["v"][sl], base["g"][sl],
+                                           base["w"][sl], 100 + shift)], 4, HP)
+    torch.cuda.synchronize()
+    ref = dict(p=t["p"][sl].copy(), m=t["m"][sl].copy(), v=t["v"][sl].copy())
+    wv, dref = oracle.commit(ref["p"], ref["m"], ref["v"], np.ascontiguousarray(t["g"][sl]), 100 + shift,
+                             oracle.resolve_hparams(HP, 4))
+    for k in "pmv":
+        got = host(base[k], np.uint32)
+        assert np.array_equal(got[sl], ref[k].view(np.uint32))
+        assert np.array_equal(got[:shift], t[k][:shift].view(np.uint32))  # untouched before the slice
+    gw = host(base["w"], np.uint16)
+    assert np.array_equal(gw[sl], wv) and not gw[:shift].any()
+    assert apc.digests_to_host(out) == dref
+
+
+@pytest.mark.parametrize("pshift,gshift", [(1, 0), (0, 3), (2, 1), (3, 5)])
+def test_mutual_misalignment_runs_scalar(pshift, gshift):
+    n = 9000
+    t = gen(n + 8, 0, 5)
+    P, Mm, V = dev(t["p"]), dev(t["m"]), dev(t["v"])
+    G = dev(t["g"])
+    Wt = torch.zeros(n + 8, dtype=torch.int16, device="cuda")
+    ps, gs = slice(pshift, pshift + n), slice(gshift, gshift + n)
+    out = apc.commit_step([apc.TensorEntry(P[ps], Mm[ps], V[ps], G[gs], Wt[gs], 7)], 5, HP)
+    torch.cuda.synchronize()
+    ref = dict(p=t["p"][ps].copy(), m=t["m"][ps].copy(), v=t["v"][ps].copy())
+    wv, dref = oracle.commit(ref["p"], ref["m"], ref["v"], np.ascontiguousarray(t["g"][gs]), 7,
+                             oracle.resolve_hparams(HP, 5))
+    assert np.array_equal(host(P, np.uint32)[ps], ref["p"].view(np.uint32))
+    assert np.array_equal(host(Mm, np.uint32)[ps], ref["m"].view(np.uint32))
+    assert np.array_equal(host(V, np.uint32)[ps], ref["v"].view(np.uint32))
+    assert np.array_equal(host(Wt, np.uint16)[gs], wv)
+    assert apc.digests_to_host(out) == dref
+
+
+def test_many_tensors_several_launches():
+    """1200 ragged tensors (more than one launch's table capacity), as views
+    with gaps into shared allocations."""
+    rng = np.random.default_rng(11)
+    sizes = rng.integers(1, 3000, size=1200)
+    tensors, off = [], (1 << 32) - 1_000_000
+    for n in sizes:
+        tensors.append(gen(int(n), off, 6))
+        off += int(n)
+    assert_same(*run_small(tensors, 6))
+
+
+def test_empty_table_and_zero_length_entries():
+    out = torch.full((4,), 123, dtype=torch.int64, device="cuda")
+    apc.commit_step([], 1, HP, out=out)
+    torch.cuda.synchronize()
+    assert apc.digests_to_host(out) == [0, 0, 0, 0]
+    t = gen(1000, 50, 1)
+    devs, dgot, ref, dref = run_small([t], 1)
+    d = devs[0]
+    entries = [apc.TensorEntry(0, 0, 0, 0, 0, 0, n=0),
+               apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], 50, n=0)]
+    apc.commit_step(entries, 1, HP, out=out)
+    torch.cuda.synchronize()
+    assert apc.digests_to_host(out) == [0, 0, 0, 0]
+    # the data were not touched by the zero-length call
+    assert np.array_equal(host(d["p"], np.uint32), ref[0]["p"].view(np.uint32))
+
+
+def test_guard_bands_untouched():
+    """Canary words around every buffer stay intact (bounds of the vector
+    head, body and tail paths)."""
+    pad = 1024
+    for n, shift in ((37, 3), (4096 + 5, 1), (12345, 0)):
+        t = gen(n, 1000, 2)
+        bufs = {}
+        for k, dt in (("p", np.float32), ("m", np.float32), ("v", np.float32), ("g", np.uint16), ("w", np.uint16)):
+            a = np.full(n + 2 * pad, 0x5A5A if dt == np.uint16 else np.float32(7.25), dtype=dt)
+            if k != "w":
+                a[pad:pad + n] = t[k]
+            bufs[k] = dev(a)
+        sl = slice(pad, pad + n)
+        apc.commit_step([apc.TensorEntry(bufs["p"][sl], bufs["m"][sl], bufs["v"][sl], bufs["g"][sl],
+                                         bufs["w"][sl], 1000)], 2, HP)
+        torch.cuda.synchronize()
+        for k in "pmv":
+            a = host(bufs[k], np.float32)
+            assert np.all(a[:pad] == np.float32(7.25)) and np.all(a[pad + n:] == np.float32(7.25))
+        for k in "gw":
+            a = host(bufs[k], np.uint16)
+            assert np.all(a[:pad] == 0x5A5A) and np.all(a[pad + n:] == 0x5A5A)
+
+
+def test_digest_of_arbitrary_buffers():
+    rng = np.random.default_rng(12)
+    bufs, want, keep = [], [0] * 8, []
+    for i in range(1100):                       # more than one launch's capacity
+        n = int(rng.integers(0, 700))
+        goff = int(rng.integers(0, 1 << 34))
+        slot = int(rng.integers(0, 8))
+        f32 = bool(rng.integers(0, 2))
+        shift = int(rng.integers(0, 8))
+        if f32:
+            a = rng.integers(0, 2**32, size=n + shift, dtype=np.uint64).astype(np.uint32)
+            t = torch.from_numpy(a.view(np.int32)).cuda()
+            want[slot] = (want[slot] + oracle.digest_f32(a[shift:], goff)) & M64
+        else:
+            a = rng.integers(0, 2**16, size=n + shift, dtype=np.uint64).astype(np.uint16)
+            t = torch.from_numpy(a.view(np.int16)).cuda()
+            want[slot] = (want[slot] + oracle.digest_u16(a[shift:], goff)) & M64
+        keep.append(t)
+        bufs.append(apc.BufferEntry(t[shift:], slot, goff, apc.F32 if f32 else apc.BF16))
+    out = apc.digest(bufs, 8)
+    assert apc.digests_to_host(out) == want
+
+
+def test_invalid_arguments_are_rejected():
+    t = gen(64, 0, 1)
+    d = dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=dev(t["g"]),
+             w=torch.zeros(64, dtype=torch.int16, device="cuda"))
+    e = apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], 0)
+    with pytest.raises(apc.ApcError) as ei:
+        apc.commit_step([e], 0, HP)
+    assert ei.value.status == 1
+    with pytest.raises(apc.ApcError) as ei:
+        apc.commit_step([e, e], 1, HP)          # the same outputs twice overlap
+    assert ei.value.status == 1
+    with pytest.raises(apc.ApcError) as ei:
+        apc.commit_step([apc.TensorEntry(d["p"].data_ptr() + 2, d["m"], d["v"], d["g"], d["w"], 0, n=8)], 1, HP)
+    assert ei.value.status == 2
+    with pytest.raises(apc.ApcError) as ei:
+        apc.commit_step([apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], M64 - 10)], 1, HP)
+    assert ei.value.status == 3
+    # nothing ran: the state is the generated one
+    assert np.array_equal(host(d["p"], np.uint32), t["p"].view(np.uint32))
+
+
+def check_sampled(dw: DeviceWorkload, step: int, k: int, seed: int):
+    idx = sample_indices(dw.w, k, seed)
+    got = dw.gather(idx)
+    ref = oracle_at(idx, step)
+    for key in "pmvw":
+        bad = np.nonzero(got[key] != ref[key])[0]
+        assert bad.size == 0, "%s differs at global %s" % (key, idx[bad[:5]])
+
+
+@pytest.mark.parametrize("step", [1, 1000])
+def test_c2_full_size(step):
+    """Mistral-7B MLP unit, 176,160,768 elements, steps 1 and 1000 from the
+    generated state: full digests against the streamed oracle and sampled
+    elements bit for bit."""
+    w = W.c2()
+    dw = DeviceWorkload(w, step)
+    out = apc.commit_step(dw.entries(), step, HP)
+    got = apc.digests_to_host(out)
+    check_sampled(dw, step, 100000, step)
+    assert got == oracle_workload_digest(w, step)
+    assert apc.digests_to_host(apc.digest(dw.digest_buffers(), 4)) == got
+    del dw
+    torch.cuda.empty_cache()
+
+
+def test_c3_full_size():
+    w = W.c3()
+    dw = DeviceWorkload(w, 10)
+    got = apc.digests_to_host(apc.commit_step(dw.entries(), 10, HP))
+    check_sampled(dw, 10, 100000, 3)
+    assert got == oracle_workload_digest(w, 10)
+    del dw
+    torch.cuda.empty_cache()
+
+
+def test_c4_rank_shard_pieces_equal_one_entry():
+    """Rank 9 of 16 (crosses 2^32): the 21-piece table and the single entry
+    give identical bits and digests, equal to the streamed oracle; the verify
+    pass reproduces the fused digests."""
+    wp, w1 = W.c4(), W.c4(one_entry=True)
+    a = DeviceWorkload(wp, 5)
+    da = apc.digests_to_host(apc.commit_step(a.entries(), 5, HP))
+    check_sampled(a, 5, 100000, 4)
+    pa = a.bufs[0]["p"].clone()
+    del a
+    b = DeviceWorkload(w1, 5)
+    db = apc.digests_to_host(apc.commit_step(b.entries(), 5, HP))
+    assert torch.equal(pa.view(torch.int32), b.bufs[0]["p"].view(torch.int32))
+    assert da == db
+    assert apc.digests_to_host(apc.digest(b.digest_buffers(), 4)) == db
+    del pa, b
+    torch.cuda.empty_cache()
+    assert da == oracle_workload_digest(wp, 5)
+
+
+def test_c5_full_model_bench_configuration():
+    """The benchmark's workload: all 291 Mistral-7B tensors (7,248,023,552
+    elements) in separate allocations, step 18, the same table and launch
+    configuration as bench.py.  Sampled elements against the oracle; the
+    verify pass equals the fused digests; the 16 rank shards' digests sum to
+    the whole (concatenation)."""
+    w = W.c5()
+    free, total = torch.cuda.mem_get_info()
+    if free < 130 * (1 << 30):
+        pytest.skip("needs ~120 GB of free device memory")
+    dw = DeviceWorkload(w, 18)
+    got = apc.digests_to_host(apc.commit_step(dw.entries(), 18, HP))
+    check_sampled(dw, 18, 200000, 5)
+    assert apc.digests_to_host(apc.digest(dw.digest_buffers(), 4)) == got
+    total = [0, 0, 0, 0]
+    for r in range(16):
+        lo, hi = W.rank_range(r, 16)
+        bufs = []
+        for pc in w.pieces:
+            a, b = max(pc.goff, lo), min(pc.goff + pc.n, hi)
+            if a < b:
+                B = dw.bufs[pc.alloc]
+                sl = slice(a - pc.goff, b - pc.goff)
+                bufs += apc.state_buffers(B["p"][sl], B["m"][sl], B["v"][sl], B["w"][sl], a)
+        d = apc.digests_to_host(apc.digest(bufs, 4))
+        total = [(x + y) & M64 for x, y in zip(total, d)]
+    assert total == got
+    del dw
+    torch.cuda.empty_cache()
+
+
+def test_repeat_runs_identical():
+    w = W.c3()
+    res = []
+    for _ in range(3):
+        dw = DeviceWorkload(w, 10)
+        res.append(apc.digests_to_host(apc.commit_step(dw.entries(), 10, HP)))
+        del dw
+    assert res[0] == res[1] == res[2]
+    torch.cuda.empty_cache()
