@@ -11,11 +11,13 @@ than L2 (129 MB), so no flush is needed between timed steps.
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
 a bounded sample of the same workload instead.
 
-Multi-GPU (torchrun): every rank runs its own replica of the shard (the
-replication group of hybrid sharding), with no collective on the data path;
-a Gloo control plane brackets the timed region with barriers, takes the
-maximum time over ranks, and checks after timing that all replicas hold
-identical digests.
+Multi-GPU (torchrun): rank r commits its own shard -- a full-size copy of
+the workload's table at global offset r * N, so the job's flat model is the
+concatenation of the ranks' shards and per-GPU work is fixed (weak scaling).
+There is no collective on the data path.  A Gloo control plane brackets the
+timed region with barriers, takes the maximum time over ranks, and after
+timing gathers every rank's digests (the whole-model digest is their
+wrapping sum) and checks that every verification pass reproduced them.
 """
 from __future__ import annotations
 
@@ -161,13 +163,28 @@ def max_over_ranks(dist, x: float) -> float:
     return float(t.item())
 
 
-def replicas_agree(dist, digests: list[int]) -> bool:
-    """All ranks hold identical digests (the replica check of recovery)."""
+def shard_offset(rank: int, elements_per_rank: int) -> int:
+    """Global index of rank r's first element: the job's flat model is the
+    concatenation of the ranks' equally sized shards (weak scaling)."""
+    return rank * elements_per_rank
+
+
+def exchange_digests(dist, commit_digests: list[int], verify_digests: list[int]):
+    """Post-step control-plane exchange (Gloo): every rank contributes its 4
+    commit digests and whether its verification pass reproduced them.
+    Returns (whole-model digests = wrapping sum over the shards, all ranks
+    verified, per-rank digests)."""
+    mine = [[int(d) & M64 for d in commit_digests], [int(d) & M64 for d in verify_digests]]
     if dist is None:
-        return True
-    gathered = [None] * dist.get_world_size()
-    dist.all_gather_object(gathered, [int(d) & M64 for d in digests])
-    return all(g == gathered[0] for g in gathered)
+        gathered = [mine]
+    else:
+        gathered = [None] * dist.get_world_size()
+        dist.all_gather_object(gathered, mine)
+    whole = [0, 0, 0, 0]
+    for c, _ in gathered:
+        whole = [(a + b) & M64 for a, b in zip(whole, c)]
+    verified = all(c == v for c, v in gathered)
+    return whole, verified, [c for c, _ in gathered]
 
 
 # ------------------------------------------------------------- GPU arm
@@ -185,6 +202,7 @@ def run_gpu(args):
     w = W.ALL[args.workload]()
     step_t = w.steps[-1]
     N = w.n
+    base = shard_offset(rank, N)   # this rank's shard of the job's flat model
 
     # resident state: one allocation per tensor, filled by the device generator
     stream = torch.cuda.current_stream()
@@ -192,7 +210,7 @@ def run_gpu(args):
     bufs = []
     goff_of = {}
     for pc in w.pieces:
-        goff_of.setdefault(pc.alloc, pc.goff - pc.at)
+        goff_of.setdefault(pc.alloc, base + pc.goff - pc.at)
     for a, n in enumerate(w.allocs):
         b = dict(p=torch.empty(n, dtype=torch.float32, device=dev), m=torch.empty(n, dtype=torch.float32, device=dev),
                  v=torch.empty(n, dtype=torch.float32, device=dev), g=torch.empty(n, dtype=torch.int16, device=dev),
@@ -207,8 +225,8 @@ def run_gpu(args):
     for pc in w.pieces:
         b = bufs[pc.alloc]
         sl = slice(pc.at, pc.at + pc.n)
-        entries.append(apc.TensorEntry(b["p"][sl], b["m"][sl], b["v"][sl], b["g"][sl], b["w"][sl], pc.goff))
-        vbufs += apc.state_buffers(b["p"][sl], b["m"][sl], b["v"][sl], b["w"][sl], pc.goff)
+        entries.append(apc.TensorEntry(b["p"][sl], b["m"][sl], b["v"][sl], b["g"][sl], b["w"][sl], base + pc.goff))
+        vbufs += apc.state_buffers(b["p"][sl], b["m"][sl], b["v"][sl], b["w"][sl], base + pc.goff)
     out_c = torch.empty(4, dtype=torch.int64, device=dev)
     out_v = torch.empty(4, dtype=torch.int64, device=dev)
     torch.cuda.synchronize()
@@ -244,7 +262,7 @@ def run_gpu(args):
     ms_per_step = total_ms / K
     digests_c = apc.digests_to_host(out_c)
     digests_v = apc.digests_to_host(out_v)
-    agree = replicas_agree(dist, digests_c + digests_v)
+    whole, verified, _ = exchange_digests(dist, digests_c, digests_v)
 
     # end to end: the step's gradient from pinned host memory, the digests back
     e2e = None
@@ -310,7 +328,7 @@ def run_gpu(args):
         "data": "synthetic",
         "config": {"workload": "%s: full Mistral-7B shard on one GPU, %d tensors, %d elements, step %d, "
                                "commit+digest then re-verify" % (w.name, len(w.pieces), N, step_t),
-                   "elements": N, "tensors": len(w.pieces), "step": step_t, "parallelism": "replica x%d" % world,
+                   "elements": N, "tensors": len(w.pieces), "step": step_t, "parallelism": "%d ranks x one shard each (no data-path collective)" % world,
                    "l2": "inputs larger than L2 (%.0f GB resident state)" % (16 * N / 1e9)},
         "hbm_gbs_step": (COMMIT_BYTES + VERIFY_BYTES) * N / (ms_per_step * 1e-3) / 1e9,
         "commit_ms": c_ms,
@@ -324,9 +342,8 @@ def run_gpu(args):
                      "traffic": profiled_traffic("commit_kernel", w.name),
                      "algorithmic_bytes_per_launch": COMMIT_BYTES * N},
         "gpu_launches": K * (1 + (len(vbufs) + 999) // 1000),
-        "digests": ["%016x" % d for d in digests_c],
-        "verify_matches_commit": digests_c == digests_v,
-        "replica_digests_agree": agree,
+        "digests": ["%016x" % d for d in whole],
+        "verify_matches_commit": verified,
         "clocks": clk,
         "e2e": e2e,
         "cpu_baseline": cpu,

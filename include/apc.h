@@ -71,7 +71,8 @@ typedef enum apc_status {
                      overlapping outputs                                          */
   APC_EALIGN = 2, /* pointer not aligned to its element size                       */
   APC_ERANGE = 3, /* global_offset + n overflows 64 bits                           */
-  APC_ECUDA = 4   /* the CUDA runtime reported an error (launch or attribute query) */
+  APC_ECUDA = 4,  /* the CUDA runtime reported an error (launch or attribute query) */
+  APC_ETIMEOUT = 5 /* a bounded wait inside a kernel gave up (see apc_device_status) */
 } apc_status;
 
 /* Decimal AdamW hyper-parameters (double).  Valid: lr >= 0, 0 <= beta < 1,
@@ -143,6 +144,20 @@ apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slot
  * step t, in the order b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/(1-b1^t),
  * 1/sqrt(1-b2^t).  Host only; no CUDA call.  out: host, 8 floats. */
 apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t step, float out[8]);
+
+/* Device-side status of this library's kernels on the current device since
+ * the previous call: APC_OK, or APC_ETIMEOUT if a bounded wait inside a
+ * kernel gave up (the digests and updates of that launch are then incomplete;
+ * a kernel that gives up stops, drains its own copies and exits, leaving the
+ * context usable).  Synchronizes the device, reads the status word and clears
+ * it.  Returns APC_ECUDA if the CUDA runtime reports an error. */
+apc_status apc_device_status(void);
+
+/* Self-test of the bounded-wait path: launch one thread on `stream` that
+ * waits on a shared-memory barrier that nothing completes; it gives up after
+ * limit_ns nanoseconds (and at least 2^20 polls) and records APC_ETIMEOUT,
+ * which the next apc_device_status() returns.  limit_ns: 1 .. 10^10. */
+apc_status apc_selftest_wait_timeout(uint64_t limit_ns, apc_stream_t stream);
 
 /* Static description of a status code. */
 const char *apc_status_string(apc_status s);

@@ -80,6 +80,10 @@ def library():
         lib.apc_last_error.restype = ctypes.c_char_p
         lib.apc_version.argtypes = []
         lib.apc_version.restype = ctypes.c_int32
+        lib.apc_device_status.argtypes = []
+        lib.apc_device_status.restype = ctypes.c_int
+        lib.apc_selftest_wait_timeout.argtypes = [ctypes.c_uint64, vp]
+        lib.apc_selftest_wait_timeout.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -221,10 +225,22 @@ def resolve_hparams(hparams: dict | None, step: int) -> list[float]:
     return list(out)
 
 
+def device_status() -> int:
+    """Synchronize the device and return (and clear) the kernels' device
+    status: 0, or 5 (APC_ETIMEOUT) if a bounded wait inside a kernel gave up."""
+    return int(library().apc_device_status())
+
+
+def selftest_wait_timeout(limit_ns: int, stream=None) -> None:
+    """Launch the bounded-wait self-test: a wait that nothing completes gives
+    up after ``limit_ns`` and records APC_ETIMEOUT for :func:`device_status`."""
+    _check(library().apc_selftest_wait_timeout(int(limit_ns), ctypes.c_void_p(_stream(stream))))
+
+
 def state_buffers(p, m, v, w, global_offset: int = 0) -> list[BufferEntry]:
     """The four digest buffers of one tensor in commit_step's slot order."""
     return [BufferEntry(p, 0, global_offset, F32), BufferEntry(m, 1, global_offset, F32),
             BufferEntry(v, 2, global_offset, F32), BufferEntry(w, 3, global_offset, BF16)]
 
 
-__all__ += ["digests_to_host", "state_buffers"]
+__all__ += ["digests_to_host", "state_buffers", "device_status", "selftest_wait_timeout"]

@@ -1,39 +1,54 @@
 // The fused committed-step kernel: AdamW over a chunk table of ragged
-// tensors, the bf16 working copy, and the four state digests, in one pass.
+// tensors, the bf16 working copy, and the four state digests, in one pass
+// over HBM (28 bytes per element: p, m, v read and written, g read, w written).
 //
-// Work decomposition.  Each table entry's vector body is cut into tiles of
-// kCommitTile = 4096 elements; a persistent grid (a multiple of the SM count)
-// walks the launch's tile space with a grid stride, so every CTA streams
-// through many tiles and the table is read from the kernel's parameter block.
-// A thread handles kCommitUnroll 8-element vectors per tile: two 16-byte
-// loads per fp32 buffer and one 16-byte bf16 load of the gradient, issued
-// for all vectors before any arithmetic so that the loads overlap.  The
-// scalar head and tail of an entry (fewer than 8 elements each) are done by
-// the CTA that owns the entry's first tile; entries whose buffers are not
-// mutually 16-byte aligned run element-wise.
+// Warp-specialized pipeline (one persistent CTA per SM by default):
+//  * The producer warp walks the launch's tiles (kCommitTile = 4096 elements
+//    of one entry's 16-byte aligned body) and, for each, waits until a ring
+//    stage is free and issues four bulk asynchronous copies -- p, m, v (16 KB
+//    each) and g (8 KB) -- that complete on the stage's "full" mbarrier.
+//    Loads never occupy consumer registers, and up to kCommitStages tiles
+//    per CTA are in flight.
+//  * The consumer warps (16 by default) wait for a stage, read their
+//    elements from shared memory (thread t of C takes elements 4t..4t+3 and
+//    4C+4t..4C+4t+3, so both the shared-memory reads and the global stores
+//    are contiguous across the warp), release the stage to the producer, then
+//    apply AdamW, store
+//    p', m', v' and the bf16 copy with 16- and 8-byte streaming stores, and
+//    fold the four digest terms into 64-bit registers.
+//  * Elements outside the aligned bodies (entry heads and tails under 8
+//    elements, and entries whose five buffers are not mutually 16-byte
+//    aligned) are "scalar items", done afterwards by the consumers with a
+//    grid-stride loop straight from global memory.
+//  * At exit the CTA sums each digest (warp shuffles, shared memory) and adds
+//    it into the caller's output with one 64-bit atomic; addition mod 2^64 is
+//    order-free, so digests do not depend on grid size or table split.
 //
-// Digest reduction.  Each thread folds its elements into four 64-bit
-// wrapping sums in registers; at exit the CTA reduces them with warp
-// shuffles and shared memory and adds one value per digest into the
-// caller's output with a 64-bit atomic.  Addition mod 2^64 is associative
-// and commutative, so the digests do not depend on the grid, the tile
-// order or the table split.
+// Every mbarrier wait is bounded (apc_tma.cuh).  A wait that gives up sets
+// the translation unit's device status word, makes the CTA stop issuing and
+// consuming, drains the copies already issued (bounded again) and returns.
 #include <cuda_runtime.h>
 
+#include "../../include/apc.h"
 #include "apc_device.cuh"
 #include "apc_internal.h"
+#include "apc_tma.cuh"
 
 namespace apc {
 namespace {
+
+__device__ unsigned int g_commit_status;
 
 struct Acc {
   uint64_t p, m, v, w;
 };
 
-struct Vec8 {
-  float4 p0, p1, m0, m1, v0, v1;
-  uint4 g;
-};
+__device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
+
+__device__ __forceinline__ void fail_wait(int *abort_flag) {
+  atomicOr(&g_commit_status, (unsigned)APC_ETIMEOUT);
+  *(volatile int *)abort_flag = 1;
+}
 
 __device__ __forceinline__ void commit_one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
   float p = E.p[i], m = E.m[i], v = E.v[i];
@@ -49,123 +64,248 @@ __device__ __forceinline__ void commit_one(const CommitEntry &E, uint64_t i, con
   a.w += digest_term(G, w);
 }
 
-__device__ __forceinline__ void load8(const CommitEntry &E, uint64_t i, Vec8 &x) {
-  const float4 *p = reinterpret_cast<const float4 *>(E.p + i);
-  const float4 *m = reinterpret_cast<const float4 *>(E.m + i);
-  const float4 *v = reinterpret_cast<const float4 *>(E.v + i);
-  x.p0 = __ldcs(p);
-  x.p1 = __ldcs(p + 1);
-  x.m0 = __ldcs(m);
-  x.m1 = __ldcs(m + 1);
-  x.v0 = __ldcs(v);
-  x.v1 = __ldcs(v + 1);
-  x.g = __ldcs(reinterpret_cast<const uint4 *>(E.g + i));
+// Four consecutive elements from shared memory, updated and stored at p, m,
+// v, w (the element's addresses in the entry); G is its digest index.
+__device__ __forceinline__ void commit_group(float *pp, float *mp, float *vp, uint16_t *wp, uint32_t G, float4 P,
+                                             float4 M, float4 V, uint2 g2, const Scalars &s, Acc &a) {
+  float p[4] = {P.x, P.y, P.z, P.w};
+  float m[4] = {M.x, M.y, M.z, M.w};
+  float v[4] = {V.x, V.y, V.z, V.w};
+  const uint32_t gw[4] = {g2.x & 0xFFFFu, g2.x >> 16, g2.y & 0xFFFFu, g2.y >> 16};
+  uint32_t w[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) w[j] = adamw_element(p[j], m[j], v[j], gw[j], s);
+  __stcs(reinterpret_cast<float4 *>(pp), make_float4(p[0], p[1], p[2], p[3]));
+  __stcs(reinterpret_cast<float4 *>(mp), make_float4(m[0], m[1], m[2], m[3]));
+  __stcs(reinterpret_cast<float4 *>(vp), make_float4(v[0], v[1], v[2], v[3]));
+  __stcs(reinterpret_cast<uint2 *>(wp), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
+  a.p += digest_term(G, __float_as_uint(p[0])) + digest_term(G + 1, __float_as_uint(p[1]));
+  a.p += digest_term(G + 2, __float_as_uint(p[2])) + digest_term(G + 3, __float_as_uint(p[3]));
+  a.m += digest_term(G, __float_as_uint(m[0])) + digest_term(G + 1, __float_as_uint(m[1]));
+  a.m += digest_term(G + 2, __float_as_uint(m[2])) + digest_term(G + 3, __float_as_uint(m[3]));
+  a.v += digest_term(G, __float_as_uint(v[0])) + digest_term(G + 1, __float_as_uint(v[1]));
+  a.v += digest_term(G + 2, __float_as_uint(v[2])) + digest_term(G + 3, __float_as_uint(v[3]));
+  a.w += digest_term(G, w[0]) + digest_term(G + 1, w[1]);
+  a.w += digest_term(G + 2, w[2]) + digest_term(G + 3, w[3]);
 }
 
-__device__ __forceinline__ void compute_store8(const CommitEntry &E, uint64_t i, const Vec8 &x, const Scalars &s,
-                                               Acc &a) {
-  float p[8] = {x.p0.x, x.p0.y, x.p0.z, x.p0.w, x.p1.x, x.p1.y, x.p1.z, x.p1.w};
-  float m[8] = {x.m0.x, x.m0.y, x.m0.z, x.m0.w, x.m1.x, x.m1.y, x.m1.z, x.m1.w};
-  float v[8] = {x.v0.x, x.v0.y, x.v0.z, x.v0.w, x.v1.x, x.v1.y, x.v1.z, x.v1.w};
-  const uint32_t gw[4] = {x.g.x, x.g.y, x.g.z, x.g.w};
-  uint32_t w[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const uint32_t g16 = (j & 1) ? (gw[j >> 1] >> 16) : (gw[j >> 1] & 0xFFFFu);
-    w[j] = adamw_element(p[j], m[j], v[j], g16, s);
-  }
-  float4 *pp = reinterpret_cast<float4 *>(E.p + i);
-  float4 *mp = reinterpret_cast<float4 *>(E.m + i);
-  float4 *vp = reinterpret_cast<float4 *>(E.v + i);
-  __stcs(pp, make_float4(p[0], p[1], p[2], p[3]));
-  __stcs(pp + 1, make_float4(p[4], p[5], p[6], p[7]));
-  __stcs(mp, make_float4(m[0], m[1], m[2], m[3]));
-  __stcs(mp + 1, make_float4(m[4], m[5], m[6], m[7]));
-  __stcs(vp, make_float4(v[0], v[1], v[2], v[3]));
-  __stcs(vp + 1, make_float4(v[4], v[5], v[6], v[7]));
-  __stcs(reinterpret_cast<uint4 *>(E.w + i),
-         make_uint4(w[0] | (w[1] << 16), w[2] | (w[3] << 16), w[4] | (w[5] << 16), w[6] | (w[7] << 16)));
-  const uint32_t G = E.key_base + (uint32_t)i;
-#pragma unroll
-  for (int j = 0; j < 8; j += 2) {
-    a.p += digest_term(G + j, __float_as_uint(p[j])) + digest_term(G + j + 1, __float_as_uint(p[j + 1]));
-    a.m += digest_term(G + j, __float_as_uint(m[j])) + digest_term(G + j + 1, __float_as_uint(m[j + 1]));
-    a.v += digest_term(G + j, __float_as_uint(v[j])) + digest_term(G + j + 1, __float_as_uint(v[j + 1]));
-    a.w += digest_term(G + j, w[j]) + digest_term(G + j + 1, w[j + 1]);
-  }
+struct Stage {
+  float *p, *m, *v;
+  uint16_t *g;
+};
+
+__device__ __forceinline__ Stage stage_at(uint8_t *smem, int s) {
+  uint8_t *b = smem + (size_t)s * kCommitStageBytes;
+  Stage st;
+  st.p = reinterpret_cast<float *>(b);
+  st.m = reinterpret_cast<float *>(b + 4 * kCommitTile);
+  st.v = reinterpret_cast<float *>(b + 8 * kCommitTile);
+  st.g = reinterpret_cast<uint16_t *>(b + 12 * kCommitTile);
+  return st;
 }
 
 template <int MAXE>
-__global__ void __launch_bounds__(kThreads) commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan,
-                                                          unsigned long long *out) {
-  __shared__ uint64_t red[kThreads / 32];
-  const Scalars s = load_scalars(plan.h);
+__device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint32_t cur, uint64_t tile) {
+  while (cur + 1 < plan.count && tile >= plan.e[cur + 1].tile_begin) ++cur;
+  return cur;
+}
+
+template <int MAXE>
+__global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
+    commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan, unsigned long long *out) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ __align__(8) uint64_t full[kCommitStages];
+  __shared__ __align__(8) uint64_t empty[kCommitStages];
+  __shared__ uint64_t red[kCommitThreads / 32];
+  __shared__ int abort_flag;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kCommitStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kCommitConsumerWarps);
+    }
+    abort_flag = 0;
+    mbar_init_fence();
+  }
+  __syncthreads();
+
   Acc a{0, 0, 0, 0};
-  uint32_t cur = 0;
-  for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
-    while (cur + 1 < plan.count && tile >= plan.e[cur + 1].tile_begin) ++cur;
-    const CommitEntry &E = plan.e[cur];
-    const uint64_t local = tile - E.tile_begin;
-    if (E.head != kScalarMode) {
-      const uint64_t head = E.head;
-      const uint64_t vec_end = head + ((E.n - head) & ~(uint64_t)(kVec - 1));
-      const uint64_t base = head + local * kCommitTile;
-      Vec8 x[kCommitUnroll];
-      bool ok[kCommitUnroll];
+  if (warp == kCommitConsumerWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t policy = l2_evict_first();
+      uint32_t cur = 0, phase = 0;
+      int stage = 0;
+      uint64_t issued = 0;
+      for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
+        if (*(volatile int *)&abort_flag) break;
+        cur = find_tile(plan, cur, tile);
+        const CommitEntry &E = plan.e[cur];
+        const uint64_t start = E.head + (tile - E.tile_begin) * kCommitTile;
+        const uint64_t vec_end = E.head + ((E.n - E.head) & ~(uint64_t)7);
+        const uint32_t cnt = (uint32_t)umin64(kCommitTile, vec_end - start);
+        if (!mbar_wait(&empty[stage], phase ^ 1)) {
+          fail_wait(&abort_flag);
+          break;
+        }
+        const Stage st = stage_at(smem, stage);
+        mbar_arrive_expect_tx(&full[stage], cnt * 14);
+        bulk_g2s(st.p, E.p + start, cnt * 4, &full[stage], policy);
+        bulk_g2s(st.m, E.m + start, cnt * 4, &full[stage], policy);
+        bulk_g2s(st.v, E.v + start, cnt * 4, &full[stage], policy);
+        bulk_g2s(st.g, E.g + start, cnt * 2, &full[stage], policy);
+        ++issued;
+        if (++stage == kCommitStages) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+      // Drain: the last min(issued, stages) copies must have landed before
+      // the CTA may exit (normally the consumers already waited for them).
+      const int n_drain = (int)umin64(issued, (uint64_t)kCommitStages);
+      for (int k = 0; k < n_drain; ++k) {
+        if (--stage < 0) {
+          stage = kCommitStages - 1;
+          phase ^= 1;
+        }
+        if (!mbar_wait(&full[stage], phase)) atomicOr(&g_commit_status, (unsigned)APC_ETIMEOUT);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ----------------------------------------------------------- consumers
+    const Scalars s = load_scalars(plan.h);
+    const int ct = threadIdx.x;  // 0..255
+    uint32_t cur = 0, phase = 0;
+    int stage = 0;
+    for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
+      cur = find_tile(plan, cur, tile);
+      const CommitEntry &E = plan.e[cur];
+      const uint64_t start = E.head + (tile - E.tile_begin) * kCommitTile;
+      const uint64_t vec_end = E.head + ((E.n - E.head) & ~(uint64_t)7);
+      const uint32_t cnt = (uint32_t)umin64(kCommitTile, vec_end - start);
+      if (!mbar_wait(&full[stage], phase)) {
+        fail_wait(&abort_flag);
+        break;
+      }
+      if (*(volatile int *)&abort_flag) break;
+      const Stage st = stage_at(smem, stage);
+      float4 P[kCommitGroups], M[kCommitGroups], V[kCommitGroups];
+      uint2 G[kCommitGroups];
+      bool ok[kCommitGroups];
 #pragma unroll
-      for (int u = 0; u < kCommitUnroll; ++u) {
-        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
-        ok[u] = i < vec_end;
-        if (ok[u]) load8(E, i, x[u]);
+      for (int k = 0; k < kCommitGroups; ++k) {
+        const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
+        ok[k] = e < cnt;
+        if (ok[k]) {
+          P[k] = *reinterpret_cast<const float4 *>(st.p + e);
+          M[k] = *reinterpret_cast<const float4 *>(st.m + e);
+          V[k] = *reinterpret_cast<const float4 *>(st.v + e);
+          G[k] = *reinterpret_cast<const uint2 *>(st.g + e);
+        }
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[stage]);
+      // the entry's fields once per tile, in registers
+      float *const pp = E.p + start, *const mp = E.m + start, *const vp = E.v + start;
+      uint16_t *const wp = E.w + start;
+      const uint32_t G0 = E.key_base + (uint32_t)start;
 #pragma unroll
-      for (int u = 0; u < kCommitUnroll; ++u) {
-        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
-        if (ok[u]) compute_store8(E, i, x[u], s, a);
+      for (int k = 0; k < kCommitGroups; ++k) {
+        const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
+        if (ok[k]) commit_group(pp + e, mp + e, vp + e, wp + e, G0 + e, P[k], M[k], V[k], G[k], s, a);
       }
-      if (local == 0) {
-        const uint32_t t = threadIdx.x;
-        if (t < head) commit_one(E, t, s, a);
-        if (t >= 32 && t - 32 < E.n - vec_end) commit_one(E, vec_end + (t - 32), s, a);
+      if (++stage == kCommitStages) {
+        stage = 0;
+        phase ^= 1;
       }
-    } else {
-      const uint64_t base = local * kCommitTile;
-#pragma unroll 4
-      for (int k = 0; k < kVec * kCommitUnroll; ++k) {
-        const uint64_t i = base + (uint64_t)k * kThreads + threadIdx.x;
-        if (i < E.n) commit_one(E, i, s, a);
+    }
+    // scalar items: entry heads and tails, and entries without vectors
+    if (!*(volatile int *)&abort_flag) {
+      cur = 0;
+      for (uint64_t it = (uint64_t)blockIdx.x * kCommitConsumers + ct; it < plan.total_scalar;
+           it += (uint64_t)gridDim.x * kCommitConsumers) {
+        while (cur + 1 < plan.count && it >= plan.e[cur + 1].scalar_begin) ++cur;
+        const CommitEntry &E = plan.e[cur];
+        const uint64_t k = it - E.scalar_begin;
+        uint64_t i;
+        if (E.head == kScalarMode) {
+          i = k;
+        } else {
+          const uint64_t vec_end = E.head + ((E.n - E.head) & ~(uint64_t)7);
+          i = k < E.head ? k : vec_end + (k - E.head);
+        }
+        commit_one(E, i, s, a);
       }
     }
   }
+
+  const bool ok = !*(volatile int *)&abort_flag;
   uint64_t r;
-  r = cta_sum<kThreads>(a.p, red);
-  if (threadIdx.x == 0 && r) atomicAdd(&out[0], (unsigned long long)r);
-  r = cta_sum<kThreads>(a.m, red);
-  if (threadIdx.x == 0 && r) atomicAdd(&out[1], (unsigned long long)r);
-  r = cta_sum<kThreads>(a.v, red);
-  if (threadIdx.x == 0 && r) atomicAdd(&out[2], (unsigned long long)r);
-  r = cta_sum<kThreads>(a.w, red);
-  if (threadIdx.x == 0 && r) atomicAdd(&out[3], (unsigned long long)r);
+  r = cta_sum<kCommitThreads>(a.p, red);
+  if (threadIdx.x == 0 && ok && r) atomicAdd(&out[0], (unsigned long long)r);
+  r = cta_sum<kCommitThreads>(a.m, red);
+  if (threadIdx.x == 0 && ok && r) atomicAdd(&out[1], (unsigned long long)r);
+  r = cta_sum<kCommitThreads>(a.v, red);
+  if (threadIdx.x == 0 && ok && r) atomicAdd(&out[2], (unsigned long long)r);
+  r = cta_sum<kCommitThreads>(a.w, red);
+  if (threadIdx.x == 0 && ok && r) atomicAdd(&out[3], (unsigned long long)r);
+}
+
+// One thread waits on an mbarrier that nothing completes: the bounded wait
+// must give up after `limit_ns` and record APC_ETIMEOUT.
+__global__ void wait_timeout_kernel(uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  mbar_init(&bar, 1);
+  mbar_init_fence();
+  if (!mbar_wait(&bar, 0, limit_ns)) atomicOr(&g_commit_status, (unsigned)APC_ETIMEOUT);
+}
+
+template <int MAXE>
+int launch(const CommitPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
+  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kCommitSmemBytes);
+  if (e != cudaSuccess) return (int)e;
+  commit_kernel<MAXE><<<grid, kCommitThreads, kCommitSmemBytes, (cudaStream_t)stream>>>(plan, out);
+  return (int)cudaGetLastError();
+}
+
+template <int MAXE>
+int blocks_per_sm(int *out) {
+  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kCommitSmemBytes);
+  if (e != cudaSuccess) return (int)e;
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<MAXE>, kCommitThreads,
+                                                            kCommitSmemBytes);
 }
 
 }  // namespace
 
 int launch_commit_small(const CommitPlan<kCommitSmall> &plan, unsigned grid, void *stream,
                         unsigned long long *out) {
-  commit_kernel<kCommitSmall><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
-  return (int)cudaGetLastError();
+  return launch(plan, grid, stream, out);
 }
 
 int launch_commit_large(const CommitPlan<kCommitLarge> &plan, unsigned grid, void *stream,
                         unsigned long long *out) {
-  commit_kernel<kCommitLarge><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
-  return (int)cudaGetLastError();
+  return launch(plan, grid, stream, out);
 }
 
 int commit_blocks_per_sm(bool large, int *out) {
-  cudaError_t e = large ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<kCommitLarge>, kThreads, 0)
-                        : cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<kCommitSmall>, kThreads, 0);
-  return (int)e;
+  return large ? blocks_per_sm<kCommitLarge>(out) : blocks_per_sm<kCommitSmall>(out);
+}
+
+int launch_wait_timeout(uint64_t limit_ns, void *stream) {
+  wait_timeout_kernel<<<1, 1, 0, (cudaStream_t)stream>>>(limit_ns);
+  return (int)cudaGetLastError();
+}
+
+int read_commit_status(unsigned *out) {
+  cudaError_t e = cudaMemcpyFromSymbol(out, g_commit_status, sizeof(unsigned));
+  if (e != cudaSuccess) return (int)e;
+  const unsigned zero = 0;
+  return (int)cudaMemcpyToSymbol(g_commit_status, &zero, sizeof(unsigned));
 }
 
 }  // namespace apc

@@ -57,7 +57,7 @@ __device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits) {
 }
 
 // Sum of a CTA's per-thread values; the result is valid in thread 0.
-// `scratch` holds kThreads/32 words.
+// `scratch` holds THREADS/32 words.
 template <int THREADS>
 __device__ __forceinline__ uint64_t cta_sum(uint64_t x, uint64_t *scratch) {
 #pragma unroll

@@ -1,8 +1,14 @@
 // The read-only state digest over a list of buffers (the verification pass
-// after recovery).  Same tiling as the commit kernel: each buffer's 16-byte
+// after recovery): 4 (fp32) or 2 (bf16) bytes read per element and one
+// splitmix64 term per element, so the pass is bound by integer issue, not by
+// HBM.  It therefore streams straight into registers: each buffer's 16-byte
 // aligned body is cut into tiles of kDigestTile elements, a persistent grid
-// strides over the launch's tile space, and the scalar head and tail of a
-// buffer go to the CTA that owns its first tile.
+// strides over the launch's tile space, every thread issues all of its
+// kDigestUnroll 16-byte (bf16) or 32-byte (fp32) loads of a tile before
+// folding any of them, and the scalar head and tail of a buffer go to the CTA
+// that owns its first tile.  (A bulk-copy pipeline like the commit kernel's
+// measured slower here: its per-tile synchronisation costs issue slots, the
+// one resource this pass is short of.)
 //
 // A thread keeps one running 64-bit sum for the slot of the buffer it is in;
 // all threads of a CTA visit the same tiles, so slot changes are CTA-uniform

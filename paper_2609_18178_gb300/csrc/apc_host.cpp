@@ -127,6 +127,8 @@ unsigned grid_for(uint64_t tiles, int sms, int per_sm) {
   return (unsigned)std::max<uint64_t>(1, std::min(tiles, cap));
 }
 
+// Entries arrive with their tile count in tile_begin and their scalar-item
+// count in scalar_begin; each batch turns both into prefix offsets.
 template <int MAXE, typename Launch>
 apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, const float h[8], unsigned grid_cap,
                               void *stream, unsigned long long *out, Launch launch) {
@@ -135,17 +137,21 @@ apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, cons
   size_t i = 0;
   while (i < entries.size()) {
     const size_t k = std::min(entries.size() - i, (size_t)MAXE);
-    uint64_t tiles = 0;
+    uint64_t tiles = 0, scalars = 0;
     for (size_t j = 0; j < k; ++j) {
       apc::CommitEntry e = entries[i + j];
-      const uint64_t t = e.tile_begin;  // holds the entry's tile count until placed
+      const uint64_t t = e.tile_begin, sc = e.scalar_begin;
       e.tile_begin = tiles;
+      e.scalar_begin = scalars;
       tiles += t;
+      scalars += sc;
       plan->e[j] = e;
     }
     plan->count = (uint32_t)k;
     plan->total_tiles = tiles;
-    const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(tiles, grid_cap));
+    plan->total_scalar = scalars;
+    const uint64_t want = std::max<uint64_t>(tiles, (scalars + apc::kCommitConsumers - 1) / apc::kCommitConsumers);
+    const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(want, grid_cap));
     int e = launch(*plan, grid, stream, out);
     if (e) return cuda_fail(e, "commit kernel launch");
     i += k;
@@ -163,7 +169,7 @@ apc_status run_digest_batches(const std::vector<apc::DigestEntry> &entries, unsi
     uint64_t tiles = 0;
     for (size_t j = 0; j < k; ++j) {
       apc::DigestEntry e = entries[i + j];
-      const uint64_t t = e.tile_begin;
+      const uint64_t t = e.tile_begin;  // holds the entry's tile count until placed
       e.tile_begin = tiles;
       tiles += t;
       plan->e[j] = e;
@@ -234,10 +240,12 @@ APC_EXPORT apc_status apc_commit_step(const apc_tensor *table, int32_t num_tenso
       const uint64_t head = std::min<uint64_t>(h0, t.n);
       const uint64_t body = (t.n - head) / apc::kVec * apc::kVec;
       e.head = (uint32_t)head;
-      e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kCommitTile));
+      e.tile_begin = ceil_div(body, apc::kCommitTile);  // tile count until placed
+      e.scalar_begin = t.n - body;                       // head + tail items
     } else {
       e.head = apc::kScalarMode;
-      e.tile_begin = ceil_div(t.n, apc::kCommitTile);
+      e.tile_begin = 0;
+      e.scalar_begin = t.n;
     }
     entries.push_back(e);
   }
@@ -287,7 +295,7 @@ APC_EXPORT apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32
     e.slot = (uint8_t)b.slot;
     e.pad_ = 0;
     const uint64_t body = (b.n - e.head) / apc::kVec * apc::kVec;
-    e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kDigestTile));
+    e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kDigestTile));  // tile count until placed
     entries.push_back(e);
   }
   int e = (int)cudaMemsetAsync(out_digests, 0, (size_t)num_slots * sizeof(uint64_t), (cudaStream_t)stream);
@@ -304,6 +312,24 @@ APC_EXPORT apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32
                                                apc::launch_digest_large);
 }
 
+APC_EXPORT apc_status apc_device_status(void) {
+  g_last_error[0] = 0;
+  int e = (int)cudaDeviceSynchronize();
+  if (e) return cuda_fail(e, "cudaDeviceSynchronize");
+  unsigned word = 0;
+  if ((e = apc::read_commit_status(&word))) return cuda_fail(e, "reading the device status word");
+  if (word & APC_ETIMEOUT) return fail(APC_ETIMEOUT, "a bounded wait inside a kernel gave up");
+  return APC_OK;
+}
+
+APC_EXPORT apc_status apc_selftest_wait_timeout(uint64_t limit_ns, apc_stream_t stream) {
+  g_last_error[0] = 0;
+  if (limit_ns < 1 || limit_ns > 10000000000ull) return fail(APC_EINVAL, "limit_ns outside 1..1e10");
+  int e = apc::launch_wait_timeout(limit_ns, stream);
+  if (e) return cuda_fail(e, "self-test kernel launch");
+  return APC_OK;
+}
+
 APC_EXPORT const char *apc_status_string(apc_status s) {
   switch (s) {
     case APC_OK: return "APC_OK: success";
@@ -311,6 +337,7 @@ APC_EXPORT const char *apc_status_string(apc_status s) {
     case APC_EALIGN: return "APC_EALIGN: misaligned pointer";
     case APC_ERANGE: return "APC_ERANGE: index range overflow";
     case APC_ECUDA: return "APC_ECUDA: CUDA runtime error";
+    case APC_ETIMEOUT: return "APC_ETIMEOUT: a bounded wait inside a kernel gave up";
   }
   return "unknown apc_status";
 }

@@ -10,19 +10,44 @@
 
 namespace apc {
 
-constexpr int kThreads = 256;              // threads per CTA
-constexpr int kVec = 8;                    // elements per thread-vector (16-byte bf16, 2 x 16-byte fp32)
-constexpr int kCommitUnroll = 2;           // thread-vectors per thread per tile (commit)
-constexpr int kDigestUnroll = 4;           // thread-vectors per thread per tile (digest)
-constexpr uint64_t kCommitTile = (uint64_t)kThreads * kVec * kCommitUnroll;  // 4096 elements
-constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 8192 elements
+constexpr int kVec = 8;                    // vector granularity: 16 bytes of bf16, 32 bytes of fp32
 constexpr uint32_t kScalarMode = 0xFFFFFFFFu;  // `head` value of an entry run without vectors
 
-// One chunk-table entry of the commit kernel (64 bytes).
-//   head: elements [0, head) are scalar, then 16-byte vectors of 8 elements
-//         up to vec_end = head + 8 * floor((n - head) / 8), then a scalar tail;
-//         kScalarMode when the five buffers are not mutually 16-byte aligned.
-//   tile_begin: index of the entry's first tile in the launch's tile space.
+// Commit kernel: warp-specialized pipeline.  One producer warp streams each
+// tile of p, m, v (fp32) and g (bf16) into a ring of shared-memory stages with
+// bulk asynchronous copies; kCommitConsumerWarps warps compute from shared
+// memory and store straight to global memory.
+// Pipeline shape (compile-time; the defaults are the measured best on GB300).
+#ifndef APC_COMMIT_CONSUMER_WARPS
+#define APC_COMMIT_CONSUMER_WARPS 16
+#endif
+#ifndef APC_COMMIT_GROUPS
+#define APC_COMMIT_GROUPS 2
+#endif
+#ifndef APC_COMMIT_STAGES
+#define APC_COMMIT_STAGES 2
+#endif
+#ifndef APC_COMMIT_BLOCKS_PER_SM
+#define APC_COMMIT_BLOCKS_PER_SM 1
+#endif
+constexpr int kCommitConsumerWarps = APC_COMMIT_CONSUMER_WARPS;
+constexpr int kCommitConsumers = kCommitConsumerWarps * 32;
+constexpr int kCommitThreads = kCommitConsumers + 32;                   // + the producer warp
+constexpr int kCommitGroups = APC_COMMIT_GROUPS;                        // 4-element groups per thread per tile
+constexpr uint64_t kCommitTile = (uint64_t)kCommitConsumers * 4 * kCommitGroups;
+constexpr int kCommitStages = APC_COMMIT_STAGES;
+constexpr uint32_t kCommitStageBytes = (uint32_t)kCommitTile * 14;      // 12 B fp32 state + 2 B grad
+constexpr uint32_t kCommitSmemBytes = kCommitStages * kCommitStageBytes;
+constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
+static_assert(kCommitSmemBytes <= 227 * 1024, "shared memory per CTA");
+
+// One chunk-table entry of the commit kernel (72 bytes).
+//   head: elements [0, head) are scalar items, then 16-byte aligned vectors
+//         up to vec_end = head + 8 * floor((n - head) / 8) in tiles of
+//         kCommitTile, then scalar items up to n; kScalarMode when the five
+//         buffers are not mutually 16-byte aligned (all n elements scalar).
+//   tile_begin: the entry's first tile in the launch's tile space.
+//   scalar_begin: the entry's first item in the launch's scalar-item space.
 //   key_base: global_offset mod 2^32 (the digest key of element 0).
 struct CommitEntry {
   float *p, *m, *v;
@@ -30,6 +55,7 @@ struct CommitEntry {
   uint16_t *w;
   uint64_t n;
   uint64_t tile_begin;
+  uint64_t scalar_begin;
   uint32_t key_base;
   uint32_t head;
 };
@@ -38,26 +64,37 @@ template <int MAXE>
 struct CommitPlan {
   float h[8];            // b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/bc1, 1/sqrt(bc2)
   uint64_t total_tiles;
+  uint64_t total_scalar;
   uint32_t count;
   uint32_t pad_;
   CommitEntry e[MAXE];
 };
 
 constexpr int kCommitSmall = 16;
-constexpr int kCommitLarge = 480;
-static_assert(sizeof(CommitEntry) == 64, "entry layout");
+constexpr int kCommitLarge = 440;
+static_assert(sizeof(CommitEntry) == 72, "entry layout");
 static_assert(sizeof(CommitPlan<kCommitLarge>) <= 32764, "kernel parameter limit");
 
+// Digest kernel: register-staged streaming (the pass is bound by integer
+// issue, so the loads are issued straight from the compute warps: a thread
+// handles kDigestUnroll 8-element vectors per tile).
+constexpr int kThreads = 256;              // threads per CTA of the digest kernel
+constexpr int kDigestUnroll = 4;           // thread-vectors per thread per tile
+constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 8192 elements
+
 // One buffer of the digest kernel (32 bytes).
+//   head: scalar elements before the first 16-byte boundary (<= 7); then
+//         8-element vectors in tiles of kDigestTile; then a scalar tail, done
+//         by the CTA that owns the buffer's first tile.
 struct DigestEntry {
   const void *data;
   uint64_t n;
   uint64_t tile_begin;
   uint32_t key_base;
-  uint8_t head;         // scalar elements before the first 16-byte vector (<= 7)
+  uint8_t head;
   uint8_t dtype;        // 0 fp32, 1 bf16
   uint8_t slot;
-  uint8_t pad_;         // a single buffer always reaches 16-byte alignment within 7 elements
+  uint8_t pad_;
 };
 
 template <int MAXE>
@@ -74,7 +111,7 @@ static_assert(sizeof(DigestEntry) == 32, "entry layout");
 static_assert(sizeof(DigestPlan<kDigestLarge>) <= 32764, "kernel parameter limit");
 
 // Launch wrappers (apc_commit.cu, apc_digest.cu).  They return a cudaError_t
-// value and launch on `stream` with `grid` CTAs of kThreads threads.
+// value and launch on `stream` with `grid` CTAs.
 int launch_commit_small(const CommitPlan<kCommitSmall> &plan, unsigned grid, void *stream,
                         unsigned long long *out);
 int launch_commit_large(const CommitPlan<kCommitLarge> &plan, unsigned grid, void *stream,
@@ -87,5 +124,13 @@ int launch_digest_large(const DigestPlan<kDigestLarge> &plan, unsigned grid, voi
 // Resident CTAs per SM of each kernel (cudaOccupancyMaxActiveBlocksPerMultiprocessor).
 int commit_blocks_per_sm(bool large, int *out);
 int digest_blocks_per_sm(bool large, int *out);
+
+// Device status word of the kernels of one translation unit on the current
+// device: nonzero after a bounded wait gave up.  read_* copies it to the host
+// (synchronously) and clears it.
+int read_commit_status(unsigned *out);
+// Self-test of the bounded wait: one thread waits on an mbarrier that nothing
+// completes, gives up after limit_ns and records APC_ETIMEOUT.
+int launch_wait_timeout(uint64_t limit_ns, void *stream);
 
 }  // namespace apc

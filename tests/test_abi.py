@@ -34,7 +34,7 @@ def test_exports_every_declared_function():
 
 def test_status_strings():
     lib = apc.library()
-    for s in range(5):
+    for s in range(6):
         assert lib.apc_status_string(s).startswith(b"APC_")
     assert b"unknown" in lib.apc_status_string(99)
 
@@ -131,6 +131,12 @@ def test_digest_argument_checks():
     assert dig([_B(None, 16, 0, 0, 0)], 4) == 1
     assert dig([_B(BASE, 100, M64 - 10, 0, 0)], 4) == 3
     assert dig([good], 4, out=0) == 1
+
+
+def test_selftest_limit_checked():
+    lib = apc.library()
+    assert lib.apc_selftest_wait_timeout(0, None) == 1
+    assert lib.apc_selftest_wait_timeout(10**11, None) == 1
 
 
 def _no_device():

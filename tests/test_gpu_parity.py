@@ -342,3 +342,15 @@ def test_repeat_runs_identical():
         del dw
     assert res[0] == res[1] == res[2]
     torch.cuda.empty_cache()
+
+
+def test_bounded_wait_gives_up_and_context_stays_usable():
+    """A kernel wait that nothing completes expires (about 50 ms and 2^20
+    polls), records APC_ETIMEOUT, and the next committed step still runs
+    bit-exact."""
+    assert apc.device_status() == 0
+    apc.selftest_wait_timeout(50_000_000)
+    assert apc.device_status() == 5
+    assert apc.device_status() == 0          # reading clears the word
+    assert_same(*run_small([gen(5000, 123, 2)], 2))
+    assert apc.device_status() == 0

@@ -1,0 +1,100 @@
+"""The multi-rank path on CPU ranks (Gloo, world size 2): each rank commits
+its own shard (here with the oracle standing in for the device), the ranks
+bracket the step with barriers and a max-over-ranks time, then exchange their
+32-byte digests on the control plane.  The whole-model digest is the wrapping
+sum of the shard digests (concatenation), and a bit flipped on one rank's
+host copy before its verification is caught by every rank."""
+import multiprocessing as mp
+import os
+import socket
+
+import numpy as np
+import pytest
+
+SIZES = [3000, 1, 4099]            # one rank's table: ragged tensors
+PER_RANK = sum(SIZES)
+STEP = 4
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, flip_rank, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
+                      LOCAL_RANK=str(rank))
+    try:
+        import bench
+        import oracle
+        import synth
+        dist = bench.init_control_plane(world)
+        base = bench.shard_offset(rank, PER_RANK)
+        h8 = oracle.resolve_hparams(oracle.DEFAULT_HP, STEP)
+        bench.barrier(dist)
+        commit, verify, off = [0, 0, 0, 0], [0, 0, 0, 0], base
+        for n in SIZES:
+            p, m, v = synth.state(n, off, nthreads=1)
+            g = synth.grad(n, off, STEP, nthreads=1)
+            w, d = oracle.commit(p, m, v, g, off, h8)
+            commit = [(a + b) & bench.M64 for a, b in zip(commit, d)]
+            if rank == flip_rank and n == SIZES[0]:
+                p.view(np.uint32)[17] ^= np.uint32(1 << 9)      # host-side fault injection
+            dv = [oracle.digest_f32(p, off), oracle.digest_f32(m, off), oracle.digest_f32(v, off),
+                  oracle.digest_u16(w, off)]
+            verify = [(a + b) & bench.M64 for a, b in zip(verify, dv)]
+            off += n
+        t = bench.max_over_ranks(dist, float(rank + 1))
+        bench.barrier(dist)
+        whole, verified, per_rank = bench.exchange_digests(dist, commit, verify)
+        dist.destroy_process_group()
+        q.put((rank, t, whole, verified, per_rank))
+    except Exception as e:  # report to the parent instead of hanging it
+        q.put((rank, "error", repr(e), None, None))
+
+
+def _run(world, flip_rank):
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, world, port, flip_rank, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    res = [q.get(timeout=240) for _ in procs]
+    for p in procs:
+        p.join(timeout=60)
+    assert all(r[1] != "error" for r in res), res
+    return sorted(res)
+
+
+def _whole_model_digest(world):
+    import oracle
+    import synth
+    h8 = oracle.resolve_hparams(oracle.DEFAULT_HP, STEP)
+    tot, off = [0, 0, 0, 0], 0
+    for _ in range(world):
+        for n in SIZES:
+            p, m, v = synth.state(n, off, nthreads=1)
+            g = synth.grad(n, off, STEP, nthreads=1)
+            _, d = oracle.commit(p, m, v, g, off, h8)
+            tot = [(a + b) % (1 << 64) for a, b in zip(tot, d)]
+            off += n
+    return tot
+
+
+def test_two_ranks_exchange_digests():
+    res = _run(2, flip_rank=-1)
+    want = _whole_model_digest(2)
+    for rank, t, whole, verified, per_rank in res:
+        assert t == 2.0                      # max over ranks of (rank + 1)
+        assert verified
+        assert whole == want                 # concatenation: shards sum to the whole model
+        assert per_rank[0] != per_rank[1]    # distinct shards
+    assert res[0][2] == res[1][2]
+
+
+def test_host_fault_on_one_rank_is_seen_by_all():
+    res = _run(2, flip_rank=1)
+    for rank, t, whole, verified, per_rank in res:
+        assert not verified
