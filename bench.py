@@ -187,6 +187,21 @@ def exchange_digests(dist, commit_digests: list[int], verify_digests: list[int])
     return whole, verified, [c for c, _ in gathered]
 
 
+def group_pieces(sizes: list[int], n_groups: int) -> list[list[int]]:
+    """Consecutive runs of table entries with about equal element counts."""
+    total = sum(sizes)
+    groups, cur, acc = [], [], 0
+    for k, n in enumerate(sizes):
+        cur.append(k)
+        acc += n
+        if acc >= total * (len(groups) + 1) / n_groups and len(groups) < n_groups - 1:
+            groups.append(cur)
+            cur = []
+    if cur:
+        groups.append(cur)
+    return groups
+
+
 # ------------------------------------------------------------- GPU arm
 
 def run_gpu(args):
@@ -264,7 +279,11 @@ def run_gpu(args):
     digests_v = apc.digests_to_host(out_v)
     whole, verified, _ = exchange_digests(dist, digests_c, digests_v)
 
-    # end to end: the step's gradient from pinned host memory, the digests back
+    # End to end: every step brings its gradient from pinned host memory and
+    # returns the digests.  The table is cut into groups of about equal size;
+    # a copy stream moves group g's gradient while the compute stream commits
+    # and verifies group g-1 (events order each group's kernels after its
+    # copies), and the host adds the per-group digests (concatenation).
     e2e = None
     if not args.no_e2e:
         host_g = []
@@ -272,15 +291,30 @@ def run_gpu(args):
             hg = torch.empty(b["g"].numel(), dtype=torch.int16, pin_memory=True)
             hg.copy_(b["g"])
             host_g.append(hg)
-        host_out = torch.empty(8, dtype=torch.int64, pin_memory=True)
+        groups = group_pieces([pc.n for pc in w.pieces], args.e2e_groups)
+        n_groups = len(groups)
+        copy_stream = torch.cuda.Stream(device=dev)
+        outs = torch.empty(n_groups, 8, dtype=torch.int64, device=dev)
+        host_out = torch.empty(n_groups, 8, dtype=torch.int64, pin_memory=True)
+        ready = [torch.cuda.Event() for _ in range(n_groups)]
+        done = [torch.cuda.Event() for _ in range(n_groups)]
+        start_ev = torch.cuda.Event()
         torch.cuda.synchronize()
 
         def e2e_step():
-            for b, hg in zip(bufs, host_g):
-                b["g"].copy_(hg, non_blocking=True)
-            one_step()
-            host_out[:4].copy_(out_c, non_blocking=True)
-            host_out[4:].copy_(out_v, non_blocking=True)
+            start_ev.record(stream)
+            copy_stream.wait_event(start_ev)
+            for gi, idx in enumerate(groups):
+                with torch.cuda.stream(copy_stream):
+                    for k in idx:
+                        pc = w.pieces[k]
+                        bufs[pc.alloc]["g"][pc.at:pc.at + pc.n].copy_(host_g[pc.alloc][pc.at:pc.at + pc.n],
+                                                                      non_blocking=True)
+                    ready[gi].record(copy_stream)
+                stream.wait_event(ready[gi])
+                apc.commit_step([entries[k] for k in idx], step_t, HP, stream=s, out=outs[gi, :4])
+                apc.digest([vbufs[4 * k + j] for k in idx for j in range(4)], 4, stream=s, out=outs[gi, 4:])
+            host_out.copy_(outs, non_blocking=True)
 
         for _ in range(max(1, args.warmup)):
             e2e_step()
@@ -296,8 +330,11 @@ def run_gpu(args):
         torch.cuda.synchronize()
         barrier(dist)
         e2e_ms = max_over_ranks(dist, e0.elapsed_time(e1)) / ke
+        got = [[int(x) & M64 for x in row] for row in host_out.tolist()]
+        e2e_verified = all(r[:4] == r[4:] for r in got)
         e2e = {"value": world * N / (e2e_ms * 1e-3), "unit": "elements/s",
-               "h2d_bytes_per_step": 2 * N, "d2h_bytes_per_step": 64, "ms_per_step": e2e_ms, "steps": ke}
+               "h2d_bytes_per_step": 2 * N, "d2h_bytes_per_step": 64 * n_groups, "ms_per_step": e2e_ms,
+               "steps": ke, "groups": n_groups, "verify_matches_commit": e2e_verified}
         del host_g
 
     cpu = None
@@ -411,6 +448,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["c1", "c2", "c3", "c4", "c5"], default="c5")
     ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-groups", type=int, default=12)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")

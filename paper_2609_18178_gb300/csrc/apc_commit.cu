@@ -175,7 +175,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
     __syncwarp();
   } else {
     // ----------------------------------------------------------- consumers
-    const Scalars s = load_scalars(plan.h);
+    const Scalars s{plan.h};
     const int ct = threadIdx.x;  // 0..255
     uint32_t cur = 0, phase = 0;
     int stage = 0;

@@ -15,30 +15,29 @@
 
 namespace apc {
 
+// The step's eight binary32 scalars, read where they are used.  In the
+// kernels they point into the launch's __grid_constant__ parameter block, so
+// every use is a constant-bank operand and holds no register.
 struct Scalars {
-  float b1, omb1, b2, omb2, eps, decay, step, rsb2;
+  const float *h;  // b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/(1-b1^t), 1/sqrt(1-b2^t)
 };
-
-__device__ __forceinline__ Scalars load_scalars(const float *h) {
-  return Scalars{h[0], h[1], h[2], h[3], h[4], h[5], h[6], h[7]};
-}
 
 // One element: p, m, v updated in place, returns the bf16 bits of p'.
 __device__ __forceinline__ uint32_t adamw_element(float &p, float &m, float &v, uint32_t g16, const Scalars &s) {
   const float g = __uint_as_float(g16 << 16);
-  const float t1 = __fmul_rn(s.b1, m);
-  const float t2 = __fmul_rn(s.omb1, g);
+  const float t1 = __fmul_rn(s.h[0], m);
+  const float t2 = __fmul_rn(s.h[1], g);
   const float mn = __fadd_rn(t1, t2);
   const float gg = __fmul_rn(g, g);
-  const float t3 = __fmul_rn(s.b2, v);
-  const float t4 = __fmul_rn(s.omb2, gg);
+  const float t3 = __fmul_rn(s.h[2], v);
+  const float t4 = __fmul_rn(s.h[3], gg);
   const float vn = __fadd_rn(t3, t4);
   const float sq = __fsqrt_rn(vn);
-  const float t5 = __fmul_rn(sq, s.rsb2);
-  const float den = __fadd_rn(t5, s.eps);
+  const float t5 = __fmul_rn(sq, s.h[7]);
+  const float den = __fadd_rn(t5, s.h[4]);
   const float u = __fdiv_rn(mn, den);
-  const float t6 = __fmul_rn(p, s.decay);
-  const float t7 = __fmul_rn(s.step, u);
+  const float t6 = __fmul_rn(p, s.h[5]);
+  const float t7 = __fmul_rn(s.h[6], u);
   const float pn = __fsub_rn(t6, t7);
   p = pn;
   m = mn;

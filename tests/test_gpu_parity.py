@@ -354,3 +354,31 @@ def test_bounded_wait_gives_up_and_context_stays_usable():
     assert apc.device_status() == 0          # reading clears the word
     assert_same(*run_small([gen(5000, 123, 2)], 2))
     assert apc.device_status() == 0
+
+
+def adversarial(n, seed):
+    """Generated state with blocks of edge values: v = 0 with g = 0 (den =
+    eps), denormal moments, large and tiny gradients, tiny and signed-zero
+    parameters, negative-zero moments."""
+    rng = np.random.default_rng(seed)
+    t = gen(n, seed * n, seed + 1)
+    p, m, v, g = t["p"], t["m"], t["v"], t["g"]
+    k = n // 8
+    v[:k] = 0.0
+    g[:k] = 0
+    m[k:2 * k] = (rng.standard_normal(k) * 1e-38).astype(np.float32)
+    v[k:2 * k] = np.abs(rng.standard_normal(k) * 1e-41).astype(np.float32)
+    g[2 * k:3 * k] = ((rng.standard_normal(k).astype(np.float32) * np.float32(10.0)).view(np.uint32) >> 16)
+    g[3 * k:4 * k] = ((rng.standard_normal(k).astype(np.float32) * np.float32(1e-12)).view(np.uint32) >> 16)
+    p[4 * k:5 * k] = (rng.standard_normal(k) * 1e-30).astype(np.float32)
+    p[5 * k:5 * k + 64] = np.float32(-0.0)
+    m[5 * k + 64:5 * k + 128] = np.float32(-0.0)
+    g[5 * k + 128:5 * k + 192] = 0x8000          # bf16 -0
+    return t
+
+
+@pytest.mark.parametrize("hp", [HP, dict(HP, lr=0.0), dict(HP, beta1=0.0), dict(HP, weight_decay=0.0),
+                                dict(lr=1e-2, beta1=0.5, beta2=0.999, eps=1e-6, weight_decay=0.01)])
+@pytest.mark.parametrize("step", [1, 7, 1000])
+def test_hyperparameters_and_edge_values(hp, step):
+    assert_same(*run_small([adversarial(40000, step), adversarial(333, step + 1)], step, hp))
