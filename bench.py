@@ -337,6 +337,39 @@ def run_gpu(args):
                "steps": ke, "groups": n_groups, "verify_matches_commit": e2e_verified}
         del host_g
 
+    # Next rows measured beside the step: the fused commit that also zeroes
+    # the gradients (30 B/element) and the quiescence guard over the
+    # gradients (2 B/element).  Run last: they leave the gradients zeroed.
+    nxt = None
+    if not args.no_next:
+        gbufs = [apc.BufferEntry(bufs[pc.alloc]["g"][pc.at:pc.at + pc.n], 0, 0, apc.BF16) for pc in w.pieces]
+        out_n = torch.empty(1, dtype=torch.int64, device=dev)
+
+        def timed(fn, reps):
+            for _ in range(2):
+                fn()
+            torch.cuda.synchronize()
+            ms = []
+            for _ in range(reps):
+                a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a0.record(stream)
+                fn()
+                a1.record(stream)
+                torch.cuda.synchronize()
+                ms.append(a0.elapsed_time(a1))
+            return statistics.median(ms)
+
+        nz_before = apc.digests_to_host(apc.count_nonzero(gbufs, 1, stream=s, out=out_n))[0]
+        guard_ms = timed(lambda: apc.count_nonzero(gbufs, 1, stream=s, out=out_n), max(3, K))
+        zero_ms = timed(lambda: apc.commit_step(entries, step_t, HP, stream=s, out=out_c, zero_grad=True), max(3, K))
+        nz_after = apc.digests_to_host(apc.count_nonzero(gbufs, 1, stream=s, out=out_n))[0]
+        peak_n, _ = measured_peak()
+        nxt = {"f1_commit_zero_grad": {"ms": zero_ms, "gbs": 30 * N / (zero_ms * 1e-3) / 1e9,
+                                       "frac": 30 * N / (zero_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 30},
+               "f1_guard_count_nonzero": {"ms": guard_ms, "gbs": 2 * N / (guard_ms * 1e-3) / 1e9,
+                                          "frac": 2 * N / (guard_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 2,
+                                          "nonzero_before": nz_before, "nonzero_after_zeroing": nz_after}}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, step_t, args.cpu_seconds)
@@ -379,11 +412,13 @@ def run_gpu(args):
                      "traffic": profiled_traffic("commit_kernel", w.name),
                      "algorithmic_bytes_per_launch": COMMIT_BYTES * N},
         "gpu_launches": K * (1 + (len(vbufs) + 999) // 1000),
+        "gpu_launches_note": "per timed step: 1 commit_kernel + 2 digest_kernel launches (1164 buffers, 1000 per launch)",
         "digests": ["%016x" % d for d in whole],
         "verify_matches_commit": verified,
         "clocks": clk,
         "e2e": e2e,
         "cpu_baseline": cpu,
+        "next_rows": nxt,
     }
     print(json.dumps(line), flush=True)
     if dist is not None:
@@ -453,6 +488,7 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-next", action="store_true", help="skip the next-row measurements (zero-grad commit, guard)")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         print("note: at least 3 warm-up steps are required for a valid number", file=sys.stderr)

@@ -128,6 +128,20 @@ typedef struct apc_buffer {
 apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
                            int64_t step, apc_stream_t stream, uint64_t *out_digests);
 
+/* Flags of apc_commit_step_ex. */
+#define APC_COMMIT_ZERO_GRAD 1u /* also write g := +0 in the same pass (the gradient buffers are written) */
+
+/* apc_commit_step with options.  flags = 0 is apc_commit_step.  With
+ * APC_COMMIT_ZERO_GRAD the pass also zeroes every gradient element after
+ * reading it, so that on return the shard sits at a committed boundary:
+ * updates landed and flat-parameter gradients zeroed (arxiv 2609.18178,
+ * Section I).  The `g` pointers are then written despite their const type,
+ * and gradient ranges count as written ranges for the overlap check.
+ * Results (p', m', v', w, digests) are identical with and without the flag.
+ * Returns APC_EINVAL for unknown flag bits, otherwise as apc_commit_step. */
+apc_status apc_commit_step_ex(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
+                              int64_t step, uint32_t flags, apc_stream_t stream, uint64_t *out_digests);
+
 /* The state digest of a list of buffers, read only.
  *
  * bufs[0..num_bufs): buffers; each adds its elements into out_digests[slot].
@@ -139,6 +153,15 @@ apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const a
  * num_slots), APC_EALIGN, APC_ERANGE, APC_ECUDA, or APC_OK. */
 apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, apc_stream_t stream,
                       uint64_t *out_digests);
+
+/* The quiescence guard: per-slot counts of buffer words whose bit pattern
+ * is nonzero, read only (the "zero outstanding gradients" check of the
+ * recovery protocol's guard, arxiv 2609.18178 Section III-C, phase 2).
+ * Same buffer list, slots and error behaviour as apc_digest (global_offset
+ * is ignored); out_counts: device, num_slots x uint64, zeroed on `stream`
+ * first.  A -0.0 word counts as nonzero. */
+apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, apc_stream_t stream,
+                             uint64_t *out_counts);
 
 /* The eight binary32 scalars that apc_commit_step passes to the device for
  * step t, in the order b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/(1-b1^t),
@@ -166,7 +189,7 @@ const char *apc_status_string(apc_status s);
  * pointer stays valid until that thread's next apc_* call. */
 const char *apc_last_error(void);
 
-/* ABI version of this header: 1. */
+/* ABI version of this header: 2. */
 int32_t apc_version(void);
 
 #ifdef __cplusplus

@@ -77,6 +77,10 @@ def _L():
         lib.oracle_commit.restype = None
         lib.oracle_commit_mt.argtypes = [vp, vp, vp, vp, vp, u64, u64, vp, vp, ctypes.c_int]
         lib.oracle_commit_mt.restype = None
+        lib.oracle_count_nonzero_u16.argtypes = [vp, u64]
+        lib.oracle_count_nonzero_u16.restype = u64
+        lib.oracle_count_nonzero_u32.argtypes = [vp, u64]
+        lib.oracle_count_nonzero_u32.restype = u64
         _lib = lib
     return _lib
 
@@ -149,6 +153,15 @@ def commit(p, m, v, g, goff: int, h8, nthreads: int = 1):
     else:
         _L().oracle_commit(*args)
     return w, [int(x) for x in d]
+
+
+def count_nonzero(a: np.ndarray) -> int:
+    """Words of a uint16/float32/uint32 array whose bit pattern is nonzero."""
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint16:
+        return int(_L().oracle_count_nonzero_u16(a.ctypes.data, a.size))
+    assert a.dtype in (np.float32, np.uint32)
+    return int(_L().oracle_count_nonzero_u32(a.ctypes.data, a.size))
 
 
 def commit_table(tensors, h8, nthreads: int = 1):

@@ -157,6 +157,22 @@ ORACLE_EXPORT void oracle_bf16_rne_array(const float *x, uint16_t *out, uint64_t
   for (uint64_t i = 0; i < n; ++i) out[i] = oracle_bf16_rne(x[i]);
 }
 
+/* ------------------------------------------------------ quiescence guard */
+
+/* Number of words whose bit pattern is nonzero (the "zero outstanding
+ * gradients" guard of the recovery protocol, Section III-C, phase 2). */
+ORACLE_EXPORT uint64_t oracle_count_nonzero_u16(const uint16_t *x, uint64_t n) {
+  uint64_t c = 0;
+  for (uint64_t i = 0; i < n; ++i) c += x[i] != 0;
+  return c;
+}
+
+ORACLE_EXPORT uint64_t oracle_count_nonzero_u32(const uint32_t *x, uint64_t n) {
+  uint64_t c = 0;
+  for (uint64_t i = 0; i < n; ++i) c += x[i] != 0;
+  return c;
+}
+
 /* ---------------------------------------------------------- whole commit */
 
 /* The committed step over one tensor: AdamW in place, then the four digests

@@ -70,6 +70,10 @@ def library():
         vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
         lib.apc_commit_step.argtypes = [vp, i32, vp, i64, vp, vp]
         lib.apc_commit_step.restype = ctypes.c_int
+        lib.apc_commit_step_ex.argtypes = [vp, i32, vp, i64, ctypes.c_uint32, vp, vp]
+        lib.apc_commit_step_ex.restype = ctypes.c_int
+        lib.apc_count_nonzero.argtypes = [vp, i32, i32, vp, vp]
+        lib.apc_count_nonzero.restype = ctypes.c_int
         lib.apc_digest.argtypes = [vp, i32, i32, vp, vp]
         lib.apc_digest.restype = ctypes.c_int
         lib.apc_resolve_hparams.argtypes = [vp, i64, vp]
@@ -165,8 +169,14 @@ def _out(out, nslots: int, like):
     return torch.empty(nslots, dtype=torch.int64, device=dev)
 
 
-def commit_step(table: Sequence[TensorEntry], step: int, hparams: dict | None = None, stream=None, out=None):
-    """Enqueue the committed AdamW step + digest over ``table`` on ``stream``.
+COMMIT_ZERO_GRAD = 1
+
+
+def commit_step(table: Sequence[TensorEntry], step: int, hparams: dict | None = None, stream=None, out=None,
+                zero_grad: bool = False):
+    """Enqueue the committed AdamW step + digest over ``table`` on ``stream``
+    (``apc_commit_step``, or ``apc_commit_step_ex`` with
+    APC_COMMIT_ZERO_GRAD when ``zero_grad``: the gradients are also zeroed).
 
     Returns the device int64[4] tensor that receives {D_p', D_m', D_v', D_w}
     (bit patterns of the unsigned digests; see :func:`digests_to_host`)."""
@@ -184,14 +194,17 @@ def commit_step(table: Sequence[TensorEntry], step: int, hparams: dict | None = 
             first = t.p
     out = _out(out, 4, first)
     hp = _hp(hparams)
-    _check(library().apc_commit_step(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
-                                     ctypes.c_void_p(_stream(stream)), ctypes.c_void_p(_ptr(out, 8))))
+    if zero_grad:
+        _check(library().apc_commit_step_ex(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
+                                            COMMIT_ZERO_GRAD, ctypes.c_void_p(_stream(stream)),
+                                            ctypes.c_void_p(_ptr(out, 8))))
+    else:
+        _check(library().apc_commit_step(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
+                                         ctypes.c_void_p(_stream(stream)), ctypes.c_void_p(_ptr(out, 8))))
     return out
 
 
-def digest(buffers: Iterable[BufferEntry], num_slots: int = 4, stream=None, out=None):
-    """Enqueue the read-only digest of ``buffers`` into ``num_slots`` slots.
-    Returns the device int64[num_slots] output tensor."""
+def _buffers(buffers):
     buffers = list(buffers)
     arr = (_Buffer * max(1, len(buffers)))()
     first = None
@@ -206,9 +219,26 @@ def digest(buffers: Iterable[BufferEntry], num_slots: int = 4, stream=None, out=
                          int(b.slot))
         if first is None and not isinstance(b.data, int):
             first = b.data
+    return arr, len(buffers), first
+
+
+def digest(buffers: Iterable[BufferEntry], num_slots: int = 4, stream=None, out=None):
+    """Enqueue the read-only digest of ``buffers`` into ``num_slots`` slots
+    (``apc_digest``).  Returns the device int64[num_slots] output tensor."""
+    arr, n, first = _buffers(buffers)
     out = _out(out, num_slots, first)
-    _check(library().apc_digest(ctypes.addressof(arr), len(buffers), int(num_slots),
-                                ctypes.c_void_p(_stream(stream)), ctypes.c_void_p(_ptr(out, 8))))
+    _check(library().apc_digest(ctypes.addressof(arr), n, int(num_slots), ctypes.c_void_p(_stream(stream)),
+                                ctypes.c_void_p(_ptr(out, 8))))
+    return out
+
+
+def count_nonzero(buffers: Iterable[BufferEntry], num_slots: int = 1, stream=None, out=None):
+    """Enqueue the quiescence guard (``apc_count_nonzero``): per-slot counts
+    of nonzero words.  Returns the device int64[num_slots] output tensor."""
+    arr, n, first = _buffers(buffers)
+    out = _out(out, num_slots, first)
+    _check(library().apc_count_nonzero(ctypes.addressof(arr), n, int(num_slots), ctypes.c_void_p(_stream(stream)),
+                                       ctypes.c_void_p(_ptr(out, 8))))
     return out
 
 
@@ -243,4 +273,5 @@ def state_buffers(p, m, v, w, global_offset: int = 0) -> list[BufferEntry]:
             BufferEntry(v, 2, global_offset, F32), BufferEntry(w, 3, global_offset, BF16)]
 
 
-__all__ += ["digests_to_host", "state_buffers", "device_status", "selftest_wait_timeout"]
+__all__ += ["digests_to_host", "state_buffers", "device_status", "selftest_wait_timeout", "count_nonzero",
+            "COMMIT_ZERO_GRAD"]

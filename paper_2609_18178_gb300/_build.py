@@ -21,12 +21,12 @@ LIB = os.path.join(BUILD, "libapc.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # exact IEEE binary32: no contraction into FMA, IEEE divide and sqrt, denormals kept
 NUMERIC = ["-fmad=false", "-prec-div=true", "-prec-sqrt=true", "-ftz=false"]
-UNITS = ["apc_commit.cu", "apc_digest.cu", "apc_host.cpp"]
+UNITS = ["apc_commit.cu", "apc_digest.cu", "apc_guard.cu", "apc_host.cpp"]
 
 
 def sources() -> list[str]:
     out = [os.path.join(CSRC, u) for u in UNITS]
-    out += [os.path.join(CSRC, h) for h in ("apc_internal.h", "apc_device.cuh")]
+    out += [os.path.join(CSRC, h) for h in ("apc_internal.h", "apc_device.cuh", "apc_tma.cuh")]
     out.append(os.path.join(INCLUDE, "apc.h"))
     return out
 

@@ -3,13 +3,13 @@
 // over HBM (28 bytes per element: p, m, v read and written, g read, w written).
 //
 // Warp-specialized pipeline (one persistent CTA per SM by default):
-//  * The producer warp walks the launch's tiles (kCommitTile = 4096 elements
+//  * The producer warp walks the launch's tiles (kCommitTile = 4864 elements
 //    of one entry's 16-byte aligned body) and, for each, waits until a ring
-//    stage is free and issues four bulk asynchronous copies -- p, m, v (16 KB
-//    each) and g (8 KB) -- that complete on the stage's "full" mbarrier.
+//    stage is free and issues four bulk asynchronous copies -- p, m, v (19 KB
+//    each) and g (9.5 KB) -- that complete on the stage's "full" mbarrier.
 //    Loads never occupy consumer registers, and up to kCommitStages tiles
 //    per CTA are in flight.
-//  * The consumer warps (16 by default) wait for a stage, read their
+//  * The consumer warps (19 by default) wait for a stage, read their
 //    elements from shared memory (thread t of C takes elements 4t..4t+3 and
 //    4C+4t..4C+4t+3, so both the shared-memory reads and the global stores
 //    are contiguous across the warp), release the stage to the producer, then
@@ -50,9 +50,11 @@ __device__ __forceinline__ void fail_wait(int *abort_flag) {
   *(volatile int *)abort_flag = 1;
 }
 
+template <bool ZERO>
 __device__ __forceinline__ void commit_one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
   float p = E.p[i], m = E.m[i], v = E.v[i];
   const uint32_t w = adamw_element(p, m, v, (uint32_t)E.g[i], s);
+  if (ZERO) const_cast<uint16_t *>(E.g)[i] = 0;
   E.p[i] = p;
   E.m[i] = m;
   E.v[i] = v;
@@ -110,7 +112,7 @@ __device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint
   return cur;
 }
 
-template <int MAXE>
+template <int MAXE, bool ZERO>
 __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
     commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan, unsigned long long *out) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -214,7 +216,10 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
 #pragma unroll
       for (int k = 0; k < kCommitGroups; ++k) {
         const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
-        if (ok[k]) commit_group(pp + e, mp + e, vp + e, wp + e, G0 + e, P[k], M[k], V[k], G[k], s, a);
+        if (ok[k]) {
+          if (ZERO) __stcs(reinterpret_cast<uint2 *>(const_cast<uint16_t *>(E.g) + start + e), make_uint2(0u, 0u));
+          commit_group(pp + e, mp + e, vp + e, wp + e, G0 + e, P[k], M[k], V[k], G[k], s, a);
+        }
       }
       if (++stage == kCommitStages) {
         stage = 0;
@@ -236,7 +241,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
           const uint64_t vec_end = E.head + ((E.n - E.head) & ~(uint64_t)7);
           i = k < E.head ? k : vec_end + (k - E.head);
         }
-        commit_one(E, i, s, a);
+        commit_one<ZERO>(E, i, s, a);
       }
     }
   }
@@ -262,34 +267,39 @@ __global__ void wait_timeout_kernel(uint64_t limit_ns) {
   if (!mbar_wait(&bar, 0, limit_ns)) atomicOr(&g_commit_status, (unsigned)APC_ETIMEOUT);
 }
 
-template <int MAXE>
-int launch(const CommitPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
-  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+template <int MAXE, bool ZERO>
+int launch_t(const CommitPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
+  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE, ZERO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kCommitSmemBytes);
   if (e != cudaSuccess) return (int)e;
-  commit_kernel<MAXE><<<grid, kCommitThreads, kCommitSmemBytes, (cudaStream_t)stream>>>(plan, out);
+  commit_kernel<MAXE, ZERO><<<grid, kCommitThreads, kCommitSmemBytes, (cudaStream_t)stream>>>(plan, out);
   return (int)cudaGetLastError();
 }
 
 template <int MAXE>
+int launch(const CommitPlan<MAXE> &plan, bool zero_grad, unsigned grid, void *stream, unsigned long long *out) {
+  return zero_grad ? launch_t<MAXE, true>(plan, grid, stream, out) : launch_t<MAXE, false>(plan, grid, stream, out);
+}
+
+template <int MAXE>
 int blocks_per_sm(int *out) {
-  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kCommitSmemBytes);
   if (e != cudaSuccess) return (int)e;
-  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<MAXE>, kCommitThreads,
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<MAXE, false>, kCommitThreads,
                                                             kCommitSmemBytes);
 }
 
 }  // namespace
 
-int launch_commit_small(const CommitPlan<kCommitSmall> &plan, unsigned grid, void *stream,
+int launch_commit_small(const CommitPlan<kCommitSmall> &plan, bool zero_grad, unsigned grid, void *stream,
                         unsigned long long *out) {
-  return launch(plan, grid, stream, out);
+  return launch(plan, zero_grad, grid, stream, out);
 }
 
-int launch_commit_large(const CommitPlan<kCommitLarge> &plan, unsigned grid, void *stream,
+int launch_commit_large(const CommitPlan<kCommitLarge> &plan, bool zero_grad, unsigned grid, void *stream,
                         unsigned long long *out) {
-  return launch(plan, grid, stream, out);
+  return launch(plan, zero_grad, grid, stream, out);
 }
 
 int commit_blocks_per_sm(bool large, int *out) {

@@ -87,7 +87,7 @@ bool overlaps(std::vector<Range> &r) {
 
 struct Device {
   int sms = 0;
-  int commit_small = 0, commit_large = 0, digest_small = 0, digest_large = 0;
+  int commit_small = 0, commit_large = 0, digest_small = 0, digest_large = 0, count_small = 0, count_large = 0;
 };
 
 constexpr int kMaxDevices = 64;
@@ -111,6 +111,8 @@ apc_status device_info(Device *out) {
   if ((e = apc::commit_blocks_per_sm(true, &d->commit_large))) return cuda_fail(e, "occupancy query");
   if ((e = apc::digest_blocks_per_sm(false, &d->digest_small))) return cuda_fail(e, "occupancy query");
   if ((e = apc::digest_blocks_per_sm(true, &d->digest_large))) return cuda_fail(e, "occupancy query");
+  if ((e = apc::count_blocks_per_sm(false, &d->count_small))) return cuda_fail(e, "occupancy query");
+  if ((e = apc::count_blocks_per_sm(true, &d->count_large))) return cuda_fail(e, "occupancy query");
   if (dev >= 0 && dev < kMaxDevices) {
     std::lock_guard<std::mutex> lock(g_device_mu);
     if (!g_device_ready[dev].load(std::memory_order_relaxed)) {
@@ -130,8 +132,8 @@ unsigned grid_for(uint64_t tiles, int sms, int per_sm) {
 // Entries arrive with their tile count in tile_begin and their scalar-item
 // count in scalar_begin; each batch turns both into prefix offsets.
 template <int MAXE, typename Launch>
-apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, const float h[8], unsigned grid_cap,
-                              void *stream, unsigned long long *out, Launch launch) {
+apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, const float h[8], bool zero_grad,
+                              unsigned grid_cap, void *stream, unsigned long long *out, Launch launch) {
   auto plan = std::make_unique<apc::CommitPlan<MAXE>>();
   std::memcpy(plan->h, h, sizeof plan->h);
   size_t i = 0;
@@ -152,7 +154,7 @@ apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, cons
     plan->total_scalar = scalars;
     const uint64_t want = std::max<uint64_t>(tiles, (scalars + apc::kCommitConsumers - 1) / apc::kCommitConsumers);
     const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(want, grid_cap));
-    int e = launch(*plan, grid, stream, out);
+    int e = launch(*plan, zero_grad, grid, stream, out);
     if (e) return cuda_fail(e, "commit kernel launch");
     i += k;
   }
@@ -161,7 +163,7 @@ apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, cons
 
 template <int MAXE, typename Launch>
 apc_status run_digest_batches(const std::vector<apc::DigestEntry> &entries, unsigned grid_cap, void *stream,
-                              unsigned long long *out, Launch launch) {
+                              unsigned long long *out, Launch launch, const char *what) {
   auto plan = std::make_unique<apc::DigestPlan<MAXE>>();
   size_t i = 0;
   while (i < entries.size()) {
@@ -178,7 +180,7 @@ apc_status run_digest_batches(const std::vector<apc::DigestEntry> &entries, unsi
     plan->total_tiles = tiles;
     const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(tiles, grid_cap));
     int e = launch(*plan, grid, stream, out);
-    if (e) return cuda_fail(e, "digest kernel launch");
+    if (e) return cuda_fail(e, what);
     i += k;
   }
   return APC_OK;
@@ -194,9 +196,12 @@ APC_EXPORT apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t s
   return resolve(hp, step, out);
 }
 
-APC_EXPORT apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
-                                      int64_t step, apc_stream_t stream, uint64_t *out_digests) {
+APC_EXPORT apc_status apc_commit_step_ex(const apc_tensor *table, int32_t num_tensors,
+                                         const apc_adamw_hparams *hp, int64_t step, uint32_t flags,
+                                         apc_stream_t stream, uint64_t *out_digests) {
   g_last_error[0] = 0;
+  if (flags & ~(uint32_t)APC_COMMIT_ZERO_GRAD) return fail(APC_EINVAL, "unknown flag bits 0x%x", flags);
+  const bool zero_grad = (flags & APC_COMMIT_ZERO_GRAD) != 0;
   if (num_tensors < 0) return fail(APC_EINVAL, "num_tensors %d < 0", num_tensors);
   if (num_tensors > 0 && !table) return fail(APC_EINVAL, "table pointer is null");
   if (!out_digests) return fail(APC_EINVAL, "out_digests pointer is null");
@@ -223,7 +228,7 @@ APC_EXPORT apc_status apc_commit_step(const apc_tensor *table, int32_t num_tenso
     ranges.push_back({m, m + 4 * t.n, true});
     ranges.push_back({v, v + 4 * t.n, true});
     ranges.push_back({w, w + 2 * t.n, true});
-    ranges.push_back({g, g + 2 * t.n, false});
+    ranges.push_back({g, g + 2 * t.n, zero_grad});
     // first element at which all five buffers sit on a 16-byte boundary
     const uint64_t h0 = ((16 - g % 16) % 16) / 2;
     const bool aligned = (p + 4 * h0) % 16 == 0 && (m + 4 * h0) % 16 == 0 && (v + 4 * h0) % 16 == 0 &&
@@ -258,23 +263,29 @@ APC_EXPORT apc_status apc_commit_step(const apc_tensor *table, int32_t num_tenso
   if ((st = device_info(&d)) != APC_OK) return st;
   unsigned long long *out = reinterpret_cast<unsigned long long *>(out_digests);
   if (entries.size() <= (size_t)apc::kCommitSmall)
-    return run_commit_batches<apc::kCommitSmall>(entries, h, grid_for(UINT64_MAX, d.sms, d.commit_small), stream,
-                                                 out, apc::launch_commit_small);
-  return run_commit_batches<apc::kCommitLarge>(entries, h, grid_for(UINT64_MAX, d.sms, d.commit_large), stream,
-                                               out, apc::launch_commit_large);
+    return run_commit_batches<apc::kCommitSmall>(entries, h, zero_grad, grid_for(UINT64_MAX, d.sms, d.commit_small),
+                                                 stream, out, apc::launch_commit_small);
+  return run_commit_batches<apc::kCommitLarge>(entries, h, zero_grad, grid_for(UINT64_MAX, d.sms, d.commit_large),
+                                               stream, out, apc::launch_commit_large);
 }
 
-APC_EXPORT apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, apc_stream_t stream,
-                                 uint64_t *out_digests) {
-  g_last_error[0] = 0;
+APC_EXPORT apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
+                                      int64_t step, apc_stream_t stream, uint64_t *out_digests) {
+  return apc_commit_step_ex(table, num_tensors, hp, step, 0u, stream, out_digests);
+}
+
+namespace {
+
+// Validate a buffer list and turn it into digest/count plan entries.
+apc_status buffer_entries(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, uint64_t *out,
+                          std::vector<apc::DigestEntry> *entries) {
   if (num_bufs < 0) return fail(APC_EINVAL, "num_bufs %d < 0", num_bufs);
   if (num_bufs > 0 && !bufs) return fail(APC_EINVAL, "bufs pointer is null");
   if (num_slots < 1 || num_slots > APC_MAX_SLOTS)
     return fail(APC_EINVAL, "num_slots %d outside 1..%d", num_slots, APC_MAX_SLOTS);
-  if (!out_digests) return fail(APC_EINVAL, "out_digests pointer is null");
-  if ((uintptr_t)out_digests % 8) return fail(APC_EALIGN, "out_digests not 8-byte aligned");
-  std::vector<apc::DigestEntry> entries;
-  entries.reserve((size_t)num_bufs);
+  if (!out) return fail(APC_EINVAL, "output pointer is null");
+  if ((uintptr_t)out % 8) return fail(APC_EALIGN, "output not 8-byte aligned");
+  entries->reserve((size_t)num_bufs);
   for (int32_t k = 0; k < num_bufs; ++k) {
     const apc_buffer &b = bufs[k];
     if (b.dtype != APC_F32 && b.dtype != APC_BF16) return fail(APC_EINVAL, "bufs[%d]: unknown dtype %u", k, b.dtype);
@@ -296,20 +307,49 @@ APC_EXPORT apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32
     e.pad_ = 0;
     const uint64_t body = (b.n - e.head) / apc::kVec * apc::kVec;
     e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kDigestTile));  // tile count until placed
-    entries.push_back(e);
+    entries->push_back(e);
   }
+  return APC_OK;
+}
+
+}  // namespace
+
+APC_EXPORT apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, apc_stream_t stream,
+                                 uint64_t *out_digests) {
+  g_last_error[0] = 0;
+  std::vector<apc::DigestEntry> entries;
+  apc_status st = buffer_entries(bufs, num_bufs, num_slots, out_digests, &entries);
+  if (st != APC_OK) return st;
   int e = (int)cudaMemsetAsync(out_digests, 0, (size_t)num_slots * sizeof(uint64_t), (cudaStream_t)stream);
   if (e) return cuda_fail(e, "cudaMemsetAsync(out_digests)");
   if (entries.empty()) return APC_OK;
   Device d;
-  apc_status st = device_info(&d);
-  if (st != APC_OK) return st;
+  if ((st = device_info(&d)) != APC_OK) return st;
   unsigned long long *out = reinterpret_cast<unsigned long long *>(out_digests);
   if (entries.size() <= (size_t)apc::kDigestSmall)
     return run_digest_batches<apc::kDigestSmall>(entries, grid_for(UINT64_MAX, d.sms, d.digest_small), stream, out,
-                                                 apc::launch_digest_small);
+                                                 apc::launch_digest_small, "digest kernel launch");
   return run_digest_batches<apc::kDigestLarge>(entries, grid_for(UINT64_MAX, d.sms, d.digest_large), stream, out,
-                                               apc::launch_digest_large);
+                                               apc::launch_digest_large, "digest kernel launch");
+}
+
+APC_EXPORT apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots,
+                                        apc_stream_t stream, uint64_t *out_counts) {
+  g_last_error[0] = 0;
+  std::vector<apc::DigestEntry> entries;
+  apc_status st = buffer_entries(bufs, num_bufs, num_slots, out_counts, &entries);
+  if (st != APC_OK) return st;
+  int e = (int)cudaMemsetAsync(out_counts, 0, (size_t)num_slots * sizeof(uint64_t), (cudaStream_t)stream);
+  if (e) return cuda_fail(e, "cudaMemsetAsync(out_counts)");
+  if (entries.empty()) return APC_OK;
+  Device d;
+  if ((st = device_info(&d)) != APC_OK) return st;
+  unsigned long long *out = reinterpret_cast<unsigned long long *>(out_counts);
+  if (entries.size() <= (size_t)apc::kDigestSmall)
+    return run_digest_batches<apc::kDigestSmall>(entries, grid_for(UINT64_MAX, d.sms, d.count_small), stream, out,
+                                                 apc::launch_count_small, "count kernel launch");
+  return run_digest_batches<apc::kDigestLarge>(entries, grid_for(UINT64_MAX, d.sms, d.count_large), stream, out,
+                                               apc::launch_count_large, "count kernel launch");
 }
 
 APC_EXPORT apc_status apc_device_status(void) {
@@ -344,4 +384,4 @@ APC_EXPORT const char *apc_status_string(apc_status s) {
 
 APC_EXPORT const char *apc_last_error(void) { return g_last_error; }
 
-APC_EXPORT int32_t apc_version(void) { return 1; }
+APC_EXPORT int32_t apc_version(void) { return 2; }

@@ -18,8 +18,12 @@ constexpr uint32_t kScalarMode = 0xFFFFFFFFu;  // `head` value of an entry run w
 // bulk asynchronous copies; kCommitConsumerWarps warps compute from shared
 // memory and store straight to global memory.
 // Pipeline shape (compile-time; the defaults are the measured best on GB300).
+// 19 consumer warps + 1 producer = 20 warps, 5 per SM sub-partition: each
+// sub-partition's 16,384 registers then give 96 per thread with no spills,
+// the same budget as 16 + 1 warps (whose fifth warp on one sub-partition sets
+// the cap), with three more warps issuing.
 #ifndef APC_COMMIT_CONSUMER_WARPS
-#define APC_COMMIT_CONSUMER_WARPS 16
+#define APC_COMMIT_CONSUMER_WARPS 19
 #endif
 #ifndef APC_COMMIT_GROUPS
 #define APC_COMMIT_GROUPS 2
@@ -112,9 +116,9 @@ static_assert(sizeof(DigestPlan<kDigestLarge>) <= 32764, "kernel parameter limit
 
 // Launch wrappers (apc_commit.cu, apc_digest.cu).  They return a cudaError_t
 // value and launch on `stream` with `grid` CTAs.
-int launch_commit_small(const CommitPlan<kCommitSmall> &plan, unsigned grid, void *stream,
+int launch_commit_small(const CommitPlan<kCommitSmall> &plan, bool zero_grad, unsigned grid, void *stream,
                         unsigned long long *out);
-int launch_commit_large(const CommitPlan<kCommitLarge> &plan, unsigned grid, void *stream,
+int launch_commit_large(const CommitPlan<kCommitLarge> &plan, bool zero_grad, unsigned grid, void *stream,
                         unsigned long long *out);
 int launch_digest_small(const DigestPlan<kDigestSmall> &plan, unsigned grid, void *stream,
                         unsigned long long *out);
@@ -124,6 +128,12 @@ int launch_digest_large(const DigestPlan<kDigestLarge> &plan, unsigned grid, voi
 // Resident CTAs per SM of each kernel (cudaOccupancyMaxActiveBlocksPerMultiprocessor).
 int commit_blocks_per_sm(bool large, int *out);
 int digest_blocks_per_sm(bool large, int *out);
+
+// Count kernel (apc_guard.cu): per-slot counts of nonzero words over the
+// same buffer plans as the digest.
+int launch_count_small(const DigestPlan<kDigestSmall> &plan, unsigned grid, void *stream, unsigned long long *out);
+int launch_count_large(const DigestPlan<kDigestLarge> &plan, unsigned grid, void *stream, unsigned long long *out);
+int count_blocks_per_sm(bool large, int *out);
 
 // Device status word of the kernels of one translation unit on the current
 // device: nonzero after a bounded wait gave up.  read_* copies it to the host

@@ -29,7 +29,7 @@ def test_exports_every_declared_function():
     lib = ctypes.CDLL(apc.lib_path() if os.path.exists(apc.lib_path()) else apc._build.build())
     for n in names:
         assert hasattr(lib, n), n
-    assert apc.library().apc_version() == 1
+    assert apc.library().apc_version() == 2
 
 
 def test_status_strings():
@@ -159,3 +159,31 @@ def test_shared_gradient_is_not_an_overlap():
     a = fake(100)
     c = fake(100, p=4000, m=(1 << 30) + 4000, v=(2 << 30) + 4000, g=(3 << 30), w=(4 << 30) + 4000)
     assert commit([a, c]) == 4
+
+
+def test_commit_ex_flags_and_zero_grad_overlap():
+    lib = apc.library()
+    h = _hp()
+
+    def ex(table, flags):
+        arr = (_T * max(1, len(table)))(*table)
+        return lib.apc_commit_step_ex(ctypes.addressof(arr), len(table), ctypes.addressof(h), 1, flags, None,
+                                      ctypes.c_void_p(0x10000))
+
+    assert ex([fake(8)], 2) == 1                                # unknown flag bit
+    a = fake(100)
+    c = fake(100, p=4000, m=(1 << 30) + 4000, v=(2 << 30) + 4000, g=(3 << 30), w=(4 << 30) + 4000)
+    assert ex([a, c], 1) == 1                                   # zeroing makes a shared gradient a written overlap
+
+
+def test_count_nonzero_argument_checks():
+    lib = apc.library()
+
+    def cnt(bufs, slots, out=0x10000):
+        arr = (_B * max(1, len(bufs)))(*bufs)
+        return lib.apc_count_nonzero(ctypes.addressof(arr), len(bufs), slots, None, ctypes.c_void_p(out))
+
+    assert cnt([_B(BASE, 16, 0, 0, 0)], 0) == 1
+    assert cnt([_B(BASE, 16, 0, 3, 0)], 1) == 1
+    assert cnt([_B(BASE + 1, 16, 0, 1, 0)], 1) == 2
+    assert cnt([_B(BASE, 16, 0, 0, 0)], 1, out=0x10001) == 2

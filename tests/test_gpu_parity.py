@@ -382,3 +382,53 @@ def adversarial(n, seed):
 @pytest.mark.parametrize("step", [1, 7, 1000])
 def test_hyperparameters_and_edge_values(hp, step):
     assert_same(*run_small([adversarial(40000, step), adversarial(333, step + 1)], step, hp))
+
+
+def test_commit_zero_grad_reaches_committed_boundary():
+    """With APC_COMMIT_ZERO_GRAD the same pass zeroes every gradient: outputs
+    and digests equal the oracle's, the guard counts the oracle's nonzero
+    gradients before and none after."""
+    tensors = [gen(n, off, 5) for n, off in ((50000, 0), (77, 50000), (123457, 50077))]
+    want_nz = sum(oracle.count_nonzero(t["g"]) for t in tensors)
+    devs, entries = [], []
+    for t in tensors:
+        d = dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=dev(t["g"]),
+                 w=torch.zeros(t["p"].size, dtype=torch.int16, device="cuda"))
+        devs.append(d)
+        entries.append(apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], t["goff"]))
+    gb = [apc.BufferEntry(d["g"], 0, 0, apc.BF16) for d in devs]
+    before = apc.digests_to_host(apc.count_nonzero(gb, 1))
+    out = apc.commit_step(entries, 5, HP, zero_grad=True)
+    after = apc.digests_to_host(apc.count_nonzero(gb, 1))
+    torch.cuda.synchronize()
+    assert before == [want_nz] and after == [0]
+    h8 = oracle.resolve_hparams(HP, 5)
+    ref = [dict(p=t["p"].copy(), m=t["m"].copy(), v=t["v"].copy(), g=t["g"], goff=t["goff"]) for t in tensors]
+    ws, dref = oracle.commit_table(ref, h8)
+    for r, wv in zip(ref, ws):
+        r["w"] = wv
+    assert_same(devs, apc.digests_to_host(out), ref, dref)
+
+
+def test_count_nonzero_of_arbitrary_buffers():
+    rng = np.random.default_rng(31)
+    bufs, want, keep = [], [0] * 8, []
+    for i in range(1100):
+        n = int(rng.integers(0, 900))
+        slot = int(rng.integers(0, 8))
+        f32 = bool(rng.integers(0, 2))
+        shift = int(rng.integers(0, 8))
+        if f32:
+            a = rng.integers(0, 2**32, size=n + shift, dtype=np.uint64).astype(np.uint32)
+            a[rng.random(n + shift) < 0.6] = 0
+            a[rng.random(n + shift) < 0.05] = 0x80000000
+            t = torch.from_numpy(a.view(np.int32)).cuda()
+        else:
+            a = rng.integers(0, 2**16, size=n + shift, dtype=np.uint64).astype(np.uint16)
+            a[rng.random(n + shift) < 0.6] = 0
+            a[rng.random(n + shift) < 0.05] = 0x8000
+            t = torch.from_numpy(a.view(np.int16)).cuda()
+        want[slot] += oracle.count_nonzero(a[shift:])
+        keep.append(t)
+        bufs.append(apc.BufferEntry(t[shift:], slot, 0, apc.F32 if f32 else apc.BF16))
+    assert apc.digests_to_host(apc.count_nonzero(bufs, 8)) == want
