@@ -364,7 +364,32 @@ def run_gpu(args):
         zero_ms = timed(lambda: apc.commit_step(entries, step_t, HP, stream=s, out=out_c, zero_grad=True), max(3, K))
         nz_after = apc.digests_to_host(apc.count_nonzero(gbufs, 1, stream=s, out=out_n))[0]
         peak_n, _ = measured_peak()
-        nxt = {"f1_commit_zero_grad": {"ms": zero_ms, "gbs": 30 * N / (zero_ms * 1e-3) / 1e9,
+        torch.cuda.synchronize()
+        # f3: the paper's bf16-state rank shard (rank 1 of 4), committed and verified
+        w3 = W.f3()
+        N3 = w3.n
+        b3 = {k: torch.empty(N3, dtype=torch.int16, device=dev) for k in "pmvg"}
+        g3 = w3.pieces[0].goff - w3.pieces[0].at
+        for k, kind in (("p", synth.P16), ("m", synth.M16), ("v", synth.V16)):
+            synth.fill_dev(kind, b3[k].data_ptr(), N3, g3, stream=s)
+        synth.fill_dev(synth.G, b3["g"].data_ptr(), N3, g3, step=w3.steps[0], stream=s)
+        e3, v3 = [], []
+        for pc in w3.pieces:
+            sl = slice(pc.at, pc.at + pc.n)
+            e3.append(apc.TensorEntryBF16(b3["p"][sl], b3["m"][sl], b3["v"][sl], b3["g"][sl], pc.goff))
+            v3 += apc.state_buffers_bf16(b3["p"][sl], b3["m"][sl], b3["v"][sl], pc.goff)
+        out3 = torch.empty(3, dtype=torch.int64, device=dev)
+        out3v = torch.empty(3, dtype=torch.int64, device=dev)
+        f3_ms = timed(lambda: apc.commit_step_bf16(e3, w3.steps[0], HP, stream=s, out=out3), max(3, K))
+        f3v_ms = timed(lambda: apc.digest(v3, 3, stream=s, out=out3v), max(3, K))
+        f3_ok = apc.digests_to_host(out3) == apc.digests_to_host(out3v)
+        del b3
+        nxt = {"f3_commit_bf16_state": {"workload": "rank 1 of 4 of Mistral-7B, %d elements, 77 pieces, bf16 p/m/v"
+                                                    % N3, "ms": f3_ms, "gbs": 14 * N3 / (f3_ms * 1e-3) / 1e9,
+                                        "frac": 14 * N3 / (f3_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 14,
+                                        "verify_ms": f3v_ms, "verify_gbs": 6 * N3 / (f3v_ms * 1e-3) / 1e9,
+                                        "verify_matches_commit": f3_ok},
+               "f1_commit_zero_grad": {"ms": zero_ms, "gbs": 30 * N / (zero_ms * 1e-3) / 1e9,
                                        "frac": 30 * N / (zero_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 30},
                "f1_guard_count_nonzero": {"ms": guard_ms, "gbs": 2 * N / (guard_ms * 1e-3) / 1e9,
                                           "frac": 2 * N / (guard_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 2,

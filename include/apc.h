@@ -142,6 +142,28 @@ apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const a
 apc_status apc_commit_step_ex(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
                               int64_t step, uint32_t flags, apc_stream_t stream, uint64_t *out_digests);
 
+/* One entry of a bf16-state chunk table: p, m, v bf16 bits (device, n
+ * elements, read and updated in place), g bf16 bits (read; written with
+ * APC_COMMIT_ZERO_GRAD).  2-byte alignment; same skipping and overlap rules
+ * as apc_tensor. */
+typedef struct apc_tensor_bf16 {
+  uint16_t *p, *m, *v;
+  const uint16_t *g;
+  uint64_t n;
+  uint64_t global_offset;
+} apc_tensor_bf16;
+
+/* The committed step with parameters and moments kept in bf16 (the paper's
+ * own setting: "Model parameters and AdamW moments use BF16", arxiv
+ * 2609.18178 Section IV-A).  Per element: p, m, v and g are widened exactly
+ * to binary32, the update runs in the same fixed order as apc_commit_step,
+ * and p', m', v' are each rounded once to bf16 (nearest even) when stored;
+ * there is no separate working copy.  out_digests: device, 3 x uint64,
+ * written as {D_p', D_m', D_v'} over the bf16 words (zero-extended).  flags
+ * as apc_commit_step_ex.  Errors as apc_commit_step. */
+apc_status apc_commit_step_bf16(const apc_tensor_bf16 *table, int32_t num_tensors, const apc_adamw_hparams *hp,
+                                int64_t step, uint32_t flags, apc_stream_t stream, uint64_t *out_digests);
+
 /* The state digest of a list of buffers, read only.
  *
  * bufs[0..num_bufs): buffers; each adds its elements into out_digests[slot].

@@ -16,6 +16,11 @@ Abstract and Section IV-F/IV-G for the bitwise state checks):
   bf16 round-to-nearest-even copy of p', and the four digests
   ``sum_i splitmix64(((G_i mod 2^32) << 32) | bits(i)) mod 2^64`` of
   p', m', v' and the bf16 copy.
+* ``commit_bf16``: the same step with p, m, v stored in bf16 (Section IV-A
+  keeps parameters and moments in BF16): widened exactly, updated in the
+  same order, each rounded once to bf16; digests of p', m', v'.
+* ``count_nonzero``: the quiescence guard's count of nonzero words
+  (Section III-C, phase 2).
 """
 from __future__ import annotations
 
@@ -77,6 +82,10 @@ def _L():
         lib.oracle_commit.restype = None
         lib.oracle_commit_mt.argtypes = [vp, vp, vp, vp, vp, u64, u64, vp, vp, ctypes.c_int]
         lib.oracle_commit_mt.restype = None
+        lib.oracle_adamw_bf16.argtypes = [vp, vp, vp, vp, u64, vp]
+        lib.oracle_adamw_bf16.restype = None
+        lib.oracle_commit_bf16.argtypes = [vp, vp, vp, vp, u64, u64, vp, vp]
+        lib.oracle_commit_bf16.restype = None
         lib.oracle_count_nonzero_u16.argtypes = [vp, u64]
         lib.oracle_count_nonzero_u16.restype = u64
         lib.oracle_count_nonzero_u32.argtypes = [vp, u64]
@@ -153,6 +162,26 @@ def commit(p, m, v, g, goff: int, h8, nthreads: int = 1):
     else:
         _L().oracle_commit(*args)
     return w, [int(x) for x in d]
+
+
+def adamw_bf16(p, m, v, g, h8) -> None:
+    """bf16-state AdamW in place on uint16 p, m, v with uint16 grad g."""
+    n = p.size
+    assert m.size == n and v.size == n and g.size == n
+    _L().oracle_adamw_bf16(_c(p, np.uint16), _c(m, np.uint16), _c(v, np.uint16), _c(g, np.uint16), n,
+                           _c(np.ascontiguousarray(h8, dtype=np.float32), np.float32))
+
+
+def commit_bf16(p, m, v, g, goff: int, h8):
+    """bf16-state committed step over one tensor, in place.  Returns the three
+    digests [Dp', Dm', Dv'] of the written bf16 words."""
+    n = p.size
+    assert m.size == n and v.size == n and g.size == n
+    d = np.zeros(3, dtype=np.uint64)
+    h = np.ascontiguousarray(h8, dtype=np.float32)
+    _L().oracle_commit_bf16(_c(p, np.uint16), _c(m, np.uint16), _c(v, np.uint16), _c(g, np.uint16), n,
+                            int(goff) & MASK64, h.ctypes.data, d.ctypes.data)
+    return [int(x) for x in d]
 
 
 def count_nonzero(a: np.ndarray) -> int:

@@ -97,23 +97,32 @@ ORACLE_EXPORT uint16_t oracle_bf16_rne(float x) {
 
 /* ------------------------------------------------------------------ AdamW */
 
-/* One element of the step, in the fixed operation order. */
-static void adamw_one(float *p, float *m, float *v, uint16_t g16, uint16_t *w, const float h[HNUM]) {
-  float g = oracle_bf16_to_f32(g16);
-  float t1 = h[HB1] * (*m);
+/* One element of the step in the fixed operation order, in binary32:
+ * (p, m, v, g) -> (p', m', v'). */
+static void adamw_core(float p, float m, float v, float g, const float h[HNUM], float *pn_out, float *mn_out,
+                       float *vn_out) {
+  float t1 = h[HB1] * m;
   float t2 = h[HOMB1] * g;
   float mn = t1 + t2;
   float gg = g * g;
-  float t3 = h[HB2] * (*v);
+  float t3 = h[HB2] * v;
   float t4 = h[HOMB2] * gg;
   float vn = t3 + t4;
   float s = sqrtf(vn);
   float t5 = s * h[HRSB2];
   float den = t5 + h[HEPS];
   float u = mn / den;
-  float t6 = (*p) * h[HDECAY];
+  float t6 = p * h[HDECAY];
   float t7 = h[HSTEP] * u;
-  float pn = t6 - t7;
+  *pn_out = t6 - t7;
+  *mn_out = mn;
+  *vn_out = vn;
+}
+
+/* One element of the fp32-state step; w receives the bf16 copy of p'. */
+static void adamw_one(float *p, float *m, float *v, uint16_t g16, uint16_t *w, const float h[HNUM]) {
+  float pn, mn, vn;
+  adamw_core(*p, *m, *v, oracle_bf16_to_f32(g16), h, &pn, &mn, &vn);
   *p = pn;
   *m = mn;
   *v = vn;
@@ -171,6 +180,33 @@ ORACLE_EXPORT uint64_t oracle_count_nonzero_u32(const uint32_t *x, uint64_t n) {
   uint64_t c = 0;
   for (uint64_t i = 0; i < n; ++i) c += x[i] != 0;
   return c;
+}
+
+/* --------------------------------------------------------- bf16 state */
+
+/* The step with p, m, v stored in bf16 (the paper keeps parameters and AdamW
+ * moments in BF16, Section IV-A): widen exactly, run the same binary32
+ * order, round each of p', m', v' once to bf16 when storing. */
+ORACLE_EXPORT void oracle_adamw_bf16(uint16_t *p, uint16_t *m, uint16_t *v, const uint16_t *g, uint64_t n,
+                                     const float h[HNUM]) {
+  for (uint64_t i = 0; i < n; ++i) {
+    float pn, mn, vn;
+    adamw_core(oracle_bf16_to_f32(p[i]), oracle_bf16_to_f32(m[i]), oracle_bf16_to_f32(v[i]),
+               oracle_bf16_to_f32(g[i]), h, &pn, &mn, &vn);
+    p[i] = oracle_bf16_rne(pn);
+    m[i] = oracle_bf16_rne(mn);
+    v[i] = oracle_bf16_rne(vn);
+  }
+}
+
+/* bf16-state step over one tensor, then the three digests of the written
+ * words (p', m', v'), added into out[0..2] mod 2^64. */
+ORACLE_EXPORT void oracle_commit_bf16(uint16_t *p, uint16_t *m, uint16_t *v, const uint16_t *g, uint64_t n,
+                                      uint64_t goff, const float h[HNUM], uint64_t out[3]) {
+  oracle_adamw_bf16(p, m, v, g, n, h);
+  out[0] += oracle_digest_u16(p, n, goff);
+  out[1] += oracle_digest_u16(m, n, goff);
+  out[2] += oracle_digest_u16(v, n, goff);
 }
 
 /* ---------------------------------------------------------- whole commit */

@@ -38,6 +38,11 @@ class _Tensor(ctypes.Structure):
                 ("w", ctypes.c_void_p), ("n", ctypes.c_uint64), ("global_offset", ctypes.c_uint64)]
 
 
+class _TensorBF16(ctypes.Structure):
+    _fields_ = [("p", ctypes.c_void_p), ("m", ctypes.c_void_p), ("v", ctypes.c_void_p), ("g", ctypes.c_void_p),
+                ("n", ctypes.c_uint64), ("global_offset", ctypes.c_uint64)]
+
+
 class _Buffer(ctypes.Structure):
     _fields_ = [("data", ctypes.c_void_p), ("n", ctypes.c_uint64), ("global_offset", ctypes.c_uint64),
                 ("dtype", ctypes.c_uint32), ("slot", ctypes.c_uint32)]
@@ -72,6 +77,8 @@ def library():
         lib.apc_commit_step.restype = ctypes.c_int
         lib.apc_commit_step_ex.argtypes = [vp, i32, vp, i64, ctypes.c_uint32, vp, vp]
         lib.apc_commit_step_ex.restype = ctypes.c_int
+        lib.apc_commit_step_bf16.argtypes = [vp, i32, vp, i64, ctypes.c_uint32, vp, vp]
+        lib.apc_commit_step_bf16.restype = ctypes.c_int
         lib.apc_count_nonzero.argtypes = [vp, i32, i32, vp, vp]
         lib.apc_count_nonzero.restype = ctypes.c_int
         lib.apc_digest.argtypes = [vp, i32, i32, vp, vp]
@@ -151,6 +158,23 @@ class TensorEntry:
 
 
 @dataclass
+class TensorEntryBF16:
+    """One entry of a bf16-state chunk table: bf16 p, m, v (updated in
+    place) and bf16 g (read), n elements at ``global_offset``."""
+    p: object
+    m: object
+    v: object
+    g: object
+    global_offset: int = 0
+    n: int | None = None
+
+    def count(self) -> int:
+        if self.n is not None:
+            return int(self.n)
+        return int(self.p.numel())
+
+
+@dataclass
 class BufferEntry:
     """One digest buffer: ``data`` (torch tensor or pointer) of ``dtype``
     (F32 or BF16), n elements at ``global_offset``, summed into ``slot``."""
@@ -201,6 +225,29 @@ def commit_step(table: Sequence[TensorEntry], step: int, hparams: dict | None = 
     else:
         _check(library().apc_commit_step(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
                                          ctypes.c_void_p(_stream(stream)), ctypes.c_void_p(_ptr(out, 8))))
+    return out
+
+
+def commit_step_bf16(table: Sequence[TensorEntryBF16], step: int, hparams: dict | None = None, stream=None,
+                     out=None, zero_grad: bool = False):
+    """Enqueue the bf16-state committed step (``apc_commit_step_bf16``).
+    Returns the device int64[3] tensor of {D_p', D_m', D_v'}."""
+    table = list(table)
+    arr = (_TensorBF16 * max(1, len(table)))()
+    first = None
+    for i, t in enumerate(table):
+        n = t.count()
+        for name, buf in (("p", t.p), ("m", t.m), ("v", t.v), ("g", t.g)):
+            if not isinstance(buf, int) and buf is not None and buf.numel() < n:
+                raise ValueError("table[%d].%s has %d < %d elements" % (i, name, buf.numel(), n))
+        arr[i] = _TensorBF16(_ptr(t.p, 2), _ptr(t.m, 2), _ptr(t.v, 2), _ptr(t.g, 2), n, int(t.global_offset) & MASK64)
+        if first is None and not isinstance(t.p, int):
+            first = t.p
+    out = _out(out, 3, first)
+    hp = _hp(hparams)
+    _check(library().apc_commit_step_bf16(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
+                                          COMMIT_ZERO_GRAD if zero_grad else 0, ctypes.c_void_p(_stream(stream)),
+                                          ctypes.c_void_p(_ptr(out, 8))))
     return out
 
 
@@ -273,5 +320,12 @@ def state_buffers(p, m, v, w, global_offset: int = 0) -> list[BufferEntry]:
             BufferEntry(v, 2, global_offset, F32), BufferEntry(w, 3, global_offset, BF16)]
 
 
+def state_buffers_bf16(p, m, v, global_offset: int = 0) -> list[BufferEntry]:
+    """The three digest buffers of one bf16-state tensor in
+    commit_step_bf16's slot order."""
+    return [BufferEntry(p, 0, global_offset, BF16), BufferEntry(m, 1, global_offset, BF16),
+            BufferEntry(v, 2, global_offset, BF16)]
+
+
 __all__ += ["digests_to_host", "state_buffers", "device_status", "selftest_wait_timeout", "count_nonzero",
-            "COMMIT_ZERO_GRAD"]
+            "COMMIT_ZERO_GRAD", "TensorEntryBF16", "commit_step_bf16", "state_buffers_bf16"]

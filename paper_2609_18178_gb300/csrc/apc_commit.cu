@@ -1,25 +1,32 @@
 // The fused committed-step kernel: AdamW over a chunk table of ragged
-// tensors, the bf16 working copy, and the four state digests, in one pass
-// over HBM (28 bytes per element: p, m, v read and written, g read, w written).
+// tensors and the state digests, in one pass over HBM.  Two state layouts
+// share the pipeline:
+//  * F32State  -- fp32 master p and moments m, v, bf16 gradient g, and a bf16
+//    working copy w of p'; four digests (p', m', v', w); 28 bytes per element
+//    (p, m, v read and written, g read, w written).
+//  * BF16State -- p, m, v kept in bf16 (the paper's setting, arxiv 2609.18178
+//    Section IV-A "Workloads"): loaded exactly into binary32, updated in the
+//    same fixed order, rounded once to bf16 (nearest even) at the store;
+//    three digests (p', m', v'); 14 bytes per element.
+// With ZERO (APC_COMMIT_ZERO_GRAD) each gradient tile is also overwritten
+// with +0 once its copy has landed: 2 more bytes per element.
 //
 // Warp-specialized pipeline (one persistent CTA per SM by default):
 //  * The producer warp walks the launch's tiles (kCommitTile = 4864 elements
 //    of one entry's 16-byte aligned body) and, for each, waits until a ring
-//    stage is free and issues four bulk asynchronous copies -- p, m, v (19 KB
-//    each) and g (9.5 KB) -- that complete on the stage's "full" mbarrier.
-//    Loads never occupy consumer registers, and up to kCommitStages tiles
-//    per CTA are in flight.
+//    stage is free and issues four bulk asynchronous copies -- p, m, v and g
+//    -- that complete on the stage's "full" mbarrier.  Loads never occupy
+//    consumer registers, and up to kCommitStages tiles per CTA are in flight.
 //  * The consumer warps (19 by default) wait for a stage, read their
 //    elements from shared memory (thread t of C takes elements 4t..4t+3 and
 //    4C+4t..4C+4t+3, so both the shared-memory reads and the global stores
 //    are contiguous across the warp), release the stage to the producer, then
-//    apply AdamW, store
-//    p', m', v' and the bf16 copy with 16- and 8-byte streaming stores, and
-//    fold the four digest terms into 64-bit registers.
+//    apply AdamW, store the results with streaming stores, and fold the
+//    digest terms into 64-bit registers.
 //  * Elements outside the aligned bodies (entry heads and tails under 8
-//    elements, and entries whose five buffers are not mutually 16-byte
-//    aligned) are "scalar items", done afterwards by the consumers with a
-//    grid-stride loop straight from global memory.
+//    elements, and entries whose buffers are not mutually 16-byte aligned)
+//    are "scalar items", done afterwards by the consumers with a grid-stride
+//    loop straight from global memory.
 //  * At exit the CTA sums each digest (warp shuffles, shared memory) and adds
 //    it into the caller's output with one 64-bit atomic; addition mod 2^64 is
 //    order-free, so digests do not depend on grid size or table split.
@@ -50,61 +57,140 @@ __device__ __forceinline__ void fail_wait(int *abort_flag) {
   *(volatile int *)abort_flag = 1;
 }
 
-template <bool ZERO>
-__device__ __forceinline__ void commit_one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
-  float p = E.p[i], m = E.m[i], v = E.v[i];
-  const uint32_t w = adamw_element(p, m, v, (uint32_t)E.g[i], s);
-  if (ZERO) const_cast<uint16_t *>(E.g)[i] = 0;
-  E.p[i] = p;
-  E.m[i] = m;
-  E.v[i] = v;
-  E.w[i] = (uint16_t)w;
-  const uint32_t G = E.key_base + (uint32_t)i;
-  a.p += digest_term(G, __float_as_uint(p));
-  a.m += digest_term(G, __float_as_uint(m));
-  a.v += digest_term(G, __float_as_uint(v));
-  a.w += digest_term(G, w);
+__device__ __forceinline__ uint32_t bf16_rne_bits(float x) {
+  return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(x));
 }
 
-// Four consecutive elements from shared memory, updated and stored at p, m,
-// v, w (the element's addresses in the entry); G is its digest index.
-__device__ __forceinline__ void commit_group(float *pp, float *mp, float *vp, uint16_t *wp, uint32_t G, float4 P,
-                                             float4 M, float4 V, uint2 g2, const Scalars &s, Acc &a) {
-  float p[4] = {P.x, P.y, P.z, P.w};
-  float m[4] = {M.x, M.y, M.z, M.w};
-  float v[4] = {V.x, V.y, V.z, V.w};
-  const uint32_t gw[4] = {g2.x & 0xFFFFu, g2.x >> 16, g2.y & 0xFFFFu, g2.y >> 16};
-  uint32_t w[4];
+__device__ __forceinline__ float bf16_value(uint32_t h) { return __uint_as_float(h << 16); }
+
+// ------------------------------------------------------------ fp32 state
+
+struct F32State {
+  static constexpr uint32_t kES = 4;        // bytes per state element
+  static constexpr int kDigests = 4;
+  struct Regs {
+    float4 p, m, v;
+    uint2 g;
+  };
+
+  __device__ static void load(const uint8_t *st, uint32_t e, Regs &r) {
+    r.p = *reinterpret_cast<const float4 *>(st + 4 * e);
+    r.m = *reinterpret_cast<const float4 *>(st + 4 * (kCommitTile + e));
+    r.v = *reinterpret_cast<const float4 *>(st + 4 * (2 * kCommitTile + e));
+    r.g = *reinterpret_cast<const uint2 *>(st + 12 * kCommitTile + 2 * e);
+  }
+
+  // Four consecutive elements at element i of the entry; G is the digest
+  // index of the first.
+  __device__ static void compute_store(const CommitEntry &E, uint64_t i, uint32_t G, const Regs &r,
+                                       const Scalars &s, Acc &a) {
+    float p[4] = {r.p.x, r.p.y, r.p.z, r.p.w};
+    float m[4] = {r.m.x, r.m.y, r.m.z, r.m.w};
+    float v[4] = {r.v.x, r.v.y, r.v.z, r.v.w};
+    const uint32_t gw[4] = {r.g.x & 0xFFFFu, r.g.x >> 16, r.g.y & 0xFFFFu, r.g.y >> 16};
+    uint32_t w[4];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) w[j] = adamw_element(p[j], m[j], v[j], gw[j], s);
-  __stcs(reinterpret_cast<float4 *>(pp), make_float4(p[0], p[1], p[2], p[3]));
-  __stcs(reinterpret_cast<float4 *>(mp), make_float4(m[0], m[1], m[2], m[3]));
-  __stcs(reinterpret_cast<float4 *>(vp), make_float4(v[0], v[1], v[2], v[3]));
-  __stcs(reinterpret_cast<uint2 *>(wp), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
-  a.p += digest_term(G, __float_as_uint(p[0])) + digest_term(G + 1, __float_as_uint(p[1]));
-  a.p += digest_term(G + 2, __float_as_uint(p[2])) + digest_term(G + 3, __float_as_uint(p[3]));
-  a.m += digest_term(G, __float_as_uint(m[0])) + digest_term(G + 1, __float_as_uint(m[1]));
-  a.m += digest_term(G + 2, __float_as_uint(m[2])) + digest_term(G + 3, __float_as_uint(m[3]));
-  a.v += digest_term(G, __float_as_uint(v[0])) + digest_term(G + 1, __float_as_uint(v[1]));
-  a.v += digest_term(G + 2, __float_as_uint(v[2])) + digest_term(G + 3, __float_as_uint(v[3]));
-  a.w += digest_term(G, w[0]) + digest_term(G + 1, w[1]);
-  a.w += digest_term(G + 2, w[2]) + digest_term(G + 3, w[3]);
-}
+    for (int j = 0; j < 4; ++j) w[j] = adamw_element(p[j], m[j], v[j], gw[j], s);
+    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.p) + i), make_float4(p[0], p[1], p[2], p[3]));
+    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.m) + i), make_float4(m[0], m[1], m[2], m[3]));
+    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.v) + i), make_float4(v[0], v[1], v[2], v[3]));
+    __stcs(reinterpret_cast<uint2 *>(E.w + i), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
+    a.p += digest_term(G, __float_as_uint(p[0])) + digest_term(G + 1, __float_as_uint(p[1]));
+    a.p += digest_term(G + 2, __float_as_uint(p[2])) + digest_term(G + 3, __float_as_uint(p[3]));
+    a.m += digest_term(G, __float_as_uint(m[0])) + digest_term(G + 1, __float_as_uint(m[1]));
+    a.m += digest_term(G + 2, __float_as_uint(m[2])) + digest_term(G + 3, __float_as_uint(m[3]));
+    a.v += digest_term(G, __float_as_uint(v[0])) + digest_term(G + 1, __float_as_uint(v[1]));
+    a.v += digest_term(G + 2, __float_as_uint(v[2])) + digest_term(G + 3, __float_as_uint(v[3]));
+    a.w += digest_term(G, w[0]) + digest_term(G + 1, w[1]);
+    a.w += digest_term(G + 2, w[2]) + digest_term(G + 3, w[3]);
+  }
 
-struct Stage {
-  float *p, *m, *v;
-  uint16_t *g;
+  __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
+    float *P = static_cast<float *>(E.p), *M = static_cast<float *>(E.m), *V = static_cast<float *>(E.v);
+    float p = P[i], m = M[i], v = V[i];
+    const uint32_t w = adamw_element(p, m, v, (uint32_t)E.g[i], s);
+    P[i] = p;
+    M[i] = m;
+    V[i] = v;
+    E.w[i] = (uint16_t)w;
+    const uint32_t G = E.key_base + (uint32_t)i;
+    a.p += digest_term(G, __float_as_uint(p));
+    a.m += digest_term(G, __float_as_uint(m));
+    a.v += digest_term(G, __float_as_uint(v));
+    a.w += digest_term(G, w);
+  }
 };
 
-__device__ __forceinline__ Stage stage_at(uint8_t *smem, int s) {
-  uint8_t *b = smem + (size_t)s * kCommitStageBytes;
-  Stage st;
-  st.p = reinterpret_cast<float *>(b);
-  st.m = reinterpret_cast<float *>(b + 4 * kCommitTile);
-  st.v = reinterpret_cast<float *>(b + 8 * kCommitTile);
-  st.g = reinterpret_cast<uint16_t *>(b + 12 * kCommitTile);
-  return st;
+// ------------------------------------------------------------ bf16 state
+
+struct BF16State {
+  static constexpr uint32_t kES = 2;
+  static constexpr int kDigests = 3;
+  struct Regs {
+    uint2 p, m, v, g;
+  };
+
+  __device__ static void load(const uint8_t *st, uint32_t e, Regs &r) {
+    r.p = *reinterpret_cast<const uint2 *>(st + 2 * e);
+    r.m = *reinterpret_cast<const uint2 *>(st + 2 * (kCommitTile + e));
+    r.v = *reinterpret_cast<const uint2 *>(st + 2 * (2 * kCommitTile + e));
+    r.g = *reinterpret_cast<const uint2 *>(st + 6 * kCommitTile + 2 * e);
+  }
+
+  __device__ static void compute_store(const CommitEntry &E, uint64_t i, uint32_t G, const Regs &r,
+                                       const Scalars &s, Acc &a) {
+    const uint32_t pw[4] = {r.p.x & 0xFFFFu, r.p.x >> 16, r.p.y & 0xFFFFu, r.p.y >> 16};
+    const uint32_t mw[4] = {r.m.x & 0xFFFFu, r.m.x >> 16, r.m.y & 0xFFFFu, r.m.y >> 16};
+    const uint32_t vw[4] = {r.v.x & 0xFFFFu, r.v.x >> 16, r.v.y & 0xFFFFu, r.v.y >> 16};
+    const uint32_t gw[4] = {r.g.x & 0xFFFFu, r.g.x >> 16, r.g.y & 0xFFFFu, r.g.y >> 16};
+    uint32_t po[4], mo[4], vo[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      float p = bf16_value(pw[j]), m = bf16_value(mw[j]), v = bf16_value(vw[j]);
+      po[j] = adamw_element(p, m, v, gw[j], s);  // bf16 of p'
+      mo[j] = bf16_rne_bits(m);
+      vo[j] = bf16_rne_bits(v);
+    }
+    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(E.p) + i),
+           make_uint2(po[0] | (po[1] << 16), po[2] | (po[3] << 16)));
+    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(E.m) + i),
+           make_uint2(mo[0] | (mo[1] << 16), mo[2] | (mo[3] << 16)));
+    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(E.v) + i),
+           make_uint2(vo[0] | (vo[1] << 16), vo[2] | (vo[3] << 16)));
+    a.p += digest_term(G, po[0]) + digest_term(G + 1, po[1]);
+    a.p += digest_term(G + 2, po[2]) + digest_term(G + 3, po[3]);
+    a.m += digest_term(G, mo[0]) + digest_term(G + 1, mo[1]);
+    a.m += digest_term(G + 2, mo[2]) + digest_term(G + 3, mo[3]);
+    a.v += digest_term(G, vo[0]) + digest_term(G + 1, vo[1]);
+    a.v += digest_term(G + 2, vo[2]) + digest_term(G + 3, vo[3]);
+  }
+
+  __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
+    uint16_t *P = static_cast<uint16_t *>(E.p), *M = static_cast<uint16_t *>(E.m), *V = static_cast<uint16_t *>(E.v);
+    float p = bf16_value(P[i]), m = bf16_value(M[i]), v = bf16_value(V[i]);
+    const uint32_t po = adamw_element(p, m, v, (uint32_t)E.g[i], s);
+    const uint32_t mo = bf16_rne_bits(m), vo = bf16_rne_bits(v);
+    P[i] = (uint16_t)po;
+    M[i] = (uint16_t)mo;
+    V[i] = (uint16_t)vo;
+    const uint32_t G = E.key_base + (uint32_t)i;
+    a.p += digest_term(G, po);
+    a.m += digest_term(G, mo);
+    a.v += digest_term(G, vo);
+  }
+};
+
+template <class L>
+__host__ __device__ constexpr uint32_t stage_bytes() {
+  return (uint32_t)kCommitTile * (3 * L::kES + 2);
 }
+
+template <class L>
+__host__ __device__ constexpr uint32_t smem_bytes() {
+  return (uint32_t)kCommitStages * stage_bytes<L>();
+}
+
+static_assert(smem_bytes<F32State>() <= 227 * 1024, "shared memory per CTA");
 
 template <int MAXE>
 __device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint32_t cur, uint64_t tile) {
@@ -112,7 +198,7 @@ __device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint
   return cur;
 }
 
-template <int MAXE, bool ZERO>
+template <class L, int MAXE, bool ZERO>
 __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
     commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan, unsigned long long *out) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -151,12 +237,14 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
           fail_wait(&abort_flag);
           break;
         }
-        const Stage st = stage_at(smem, stage);
-        mbar_arrive_expect_tx(&full[stage], cnt * 14);
-        bulk_g2s(st.p, E.p + start, cnt * 4, &full[stage], policy);
-        bulk_g2s(st.m, E.m + start, cnt * 4, &full[stage], policy);
-        bulk_g2s(st.v, E.v + start, cnt * 4, &full[stage], policy);
-        bulk_g2s(st.g, E.g + start, cnt * 2, &full[stage], policy);
+        uint8_t *st = smem + (size_t)stage * stage_bytes<L>();
+        mbar_arrive_expect_tx(&full[stage], cnt * (3 * L::kES + 2));
+        bulk_g2s(st, static_cast<const uint8_t *>(E.p) + start * L::kES, cnt * L::kES, &full[stage], policy);
+        bulk_g2s(st + L::kES * kCommitTile, static_cast<const uint8_t *>(E.m) + start * L::kES, cnt * L::kES,
+                 &full[stage], policy);
+        bulk_g2s(st + 2 * L::kES * kCommitTile, static_cast<const uint8_t *>(E.v) + start * L::kES,
+                 cnt * L::kES, &full[stage], policy);
+        bulk_g2s(st + 3 * L::kES * kCommitTile, E.g + start, cnt * 2, &full[stage], policy);
         ++issued;
         if (++stage == kCommitStages) {
           stage = 0;
@@ -178,7 +266,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
   } else {
     // ----------------------------------------------------------- consumers
     const Scalars s{plan.h};
-    const int ct = threadIdx.x;  // 0..255
+    const int ct = threadIdx.x;  // 0 .. kCommitConsumers-1
     uint32_t cur = 0, phase = 0;
     int stage = 0;
     for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
@@ -192,33 +280,24 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
         break;
       }
       if (*(volatile int *)&abort_flag) break;
-      const Stage st = stage_at(smem, stage);
-      float4 P[kCommitGroups], M[kCommitGroups], V[kCommitGroups];
-      uint2 G[kCommitGroups];
+      const uint8_t *st = smem + (size_t)stage * stage_bytes<L>();
+      typename L::Regs r[kCommitGroups];
       bool ok[kCommitGroups];
 #pragma unroll
       for (int k = 0; k < kCommitGroups; ++k) {
         const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
         ok[k] = e < cnt;
-        if (ok[k]) {
-          P[k] = *reinterpret_cast<const float4 *>(st.p + e);
-          M[k] = *reinterpret_cast<const float4 *>(st.m + e);
-          V[k] = *reinterpret_cast<const float4 *>(st.v + e);
-          G[k] = *reinterpret_cast<const uint2 *>(st.g + e);
-        }
+        if (ok[k]) L::load(st, e, r[k]);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[stage]);
-      // the entry's fields once per tile, in registers
-      float *const pp = E.p + start, *const mp = E.m + start, *const vp = E.v + start;
-      uint16_t *const wp = E.w + start;
       const uint32_t G0 = E.key_base + (uint32_t)start;
 #pragma unroll
       for (int k = 0; k < kCommitGroups; ++k) {
         const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
         if (ok[k]) {
           if (ZERO) __stcs(reinterpret_cast<uint2 *>(const_cast<uint16_t *>(E.g) + start + e), make_uint2(0u, 0u));
-          commit_group(pp + e, mp + e, vp + e, wp + e, G0 + e, P[k], M[k], V[k], G[k], s, a);
+          L::compute_store(E, start + e, G0 + e, r[k], s, a);
         }
       }
       if (++stage == kCommitStages) {
@@ -241,7 +320,8 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
           const uint64_t vec_end = E.head + ((E.n - E.head) & ~(uint64_t)7);
           i = k < E.head ? k : vec_end + (k - E.head);
         }
-        commit_one<ZERO>(E, i, s, a);
+        L::one(E, i, s, a);
+        if (ZERO) const_cast<uint16_t *>(E.g)[i] = 0;
       }
     }
   }
@@ -254,8 +334,10 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
   if (threadIdx.x == 0 && ok && r) atomicAdd(&out[1], (unsigned long long)r);
   r = cta_sum<kCommitThreads>(a.v, red);
   if (threadIdx.x == 0 && ok && r) atomicAdd(&out[2], (unsigned long long)r);
-  r = cta_sum<kCommitThreads>(a.w, red);
-  if (threadIdx.x == 0 && ok && r) atomicAdd(&out[3], (unsigned long long)r);
+  if (L::kDigests == 4) {
+    r = cta_sum<kCommitThreads>(a.w, red);
+    if (threadIdx.x == 0 && ok && r) atomicAdd(&out[3], (unsigned long long)r);
+  }
 }
 
 // One thread waits on an mbarrier that nothing completes: the bounded wait
@@ -267,43 +349,50 @@ __global__ void wait_timeout_kernel(uint64_t limit_ns) {
   if (!mbar_wait(&bar, 0, limit_ns)) atomicOr(&g_commit_status, (unsigned)APC_ETIMEOUT);
 }
 
-template <int MAXE, bool ZERO>
+template <class L, int MAXE, bool ZERO>
 int launch_t(const CommitPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
-  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE, ZERO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kCommitSmemBytes);
+  cudaError_t e = cudaFuncSetAttribute(commit_kernel<L, MAXE, ZERO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem_bytes<L>());
   if (e != cudaSuccess) return (int)e;
-  commit_kernel<MAXE, ZERO><<<grid, kCommitThreads, kCommitSmemBytes, (cudaStream_t)stream>>>(plan, out);
+  commit_kernel<L, MAXE, ZERO><<<grid, kCommitThreads, smem_bytes<L>(), (cudaStream_t)stream>>>(plan, out);
   return (int)cudaGetLastError();
 }
 
 template <int MAXE>
-int launch(const CommitPlan<MAXE> &plan, bool zero_grad, unsigned grid, void *stream, unsigned long long *out) {
-  return zero_grad ? launch_t<MAXE, true>(plan, grid, stream, out) : launch_t<MAXE, false>(plan, grid, stream, out);
+int launch(const CommitPlan<MAXE> &plan, int layout, bool zero_grad, unsigned grid, void *stream,
+           unsigned long long *out) {
+  if (layout == kLayoutBF16)
+    return zero_grad ? launch_t<BF16State, MAXE, true>(plan, grid, stream, out)
+                     : launch_t<BF16State, MAXE, false>(plan, grid, stream, out);
+  return zero_grad ? launch_t<F32State, MAXE, true>(plan, grid, stream, out)
+                   : launch_t<F32State, MAXE, false>(plan, grid, stream, out);
 }
 
-template <int MAXE>
+template <class L, int MAXE>
 int blocks_per_sm(int *out) {
-  cudaError_t e = cudaFuncSetAttribute(commit_kernel<MAXE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kCommitSmemBytes);
+  cudaError_t e = cudaFuncSetAttribute(commit_kernel<L, MAXE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem_bytes<L>());
   if (e != cudaSuccess) return (int)e;
-  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<MAXE, false>, kCommitThreads,
-                                                            kCommitSmemBytes);
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<L, MAXE, false>, kCommitThreads,
+                                                            smem_bytes<L>());
 }
 
 }  // namespace
 
-int launch_commit_small(const CommitPlan<kCommitSmall> &plan, bool zero_grad, unsigned grid, void *stream,
-                        unsigned long long *out) {
-  return launch(plan, zero_grad, grid, stream, out);
+int launch_commit_small(const CommitPlan<kCommitSmall> &plan, int layout, bool zero_grad, unsigned grid,
+                        void *stream, unsigned long long *out) {
+  return launch(plan, layout, zero_grad, grid, stream, out);
 }
 
-int launch_commit_large(const CommitPlan<kCommitLarge> &plan, bool zero_grad, unsigned grid, void *stream,
-                        unsigned long long *out) {
-  return launch(plan, zero_grad, grid, stream, out);
+int launch_commit_large(const CommitPlan<kCommitLarge> &plan, int layout, bool zero_grad, unsigned grid,
+                        void *stream, unsigned long long *out) {
+  return launch(plan, layout, zero_grad, grid, stream, out);
 }
 
 int commit_blocks_per_sm(bool large, int *out) {
-  return large ? blocks_per_sm<kCommitLarge>(out) : blocks_per_sm<kCommitSmall>(out);
+  // the fp32 layout has the larger shared-memory footprint, so its residency
+  // also holds for the bf16 layout
+  return large ? blocks_per_sm<F32State, kCommitLarge>(out) : blocks_per_sm<F32State, kCommitSmall>(out);
 }
 
 int launch_wait_timeout(uint64_t limit_ns, void *stream) {

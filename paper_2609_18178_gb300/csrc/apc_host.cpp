@@ -132,8 +132,9 @@ unsigned grid_for(uint64_t tiles, int sms, int per_sm) {
 // Entries arrive with their tile count in tile_begin and their scalar-item
 // count in scalar_begin; each batch turns both into prefix offsets.
 template <int MAXE, typename Launch>
-apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, const float h[8], bool zero_grad,
-                              unsigned grid_cap, void *stream, unsigned long long *out, Launch launch) {
+apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, const float h[8], int layout,
+                              bool zero_grad, unsigned grid_cap, void *stream, unsigned long long *out,
+                              Launch launch) {
   auto plan = std::make_unique<apc::CommitPlan<MAXE>>();
   std::memcpy(plan->h, h, sizeof plan->h);
   size_t i = 0;
@@ -154,7 +155,7 @@ apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, cons
     plan->total_scalar = scalars;
     const uint64_t want = std::max<uint64_t>(tiles, (scalars + apc::kCommitConsumers - 1) / apc::kCommitConsumers);
     const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(want, grid_cap));
-    int e = launch(*plan, zero_grad, grid, stream, out);
+    int e = launch(*plan, layout, zero_grad, grid, stream, out);
     if (e) return cuda_fail(e, "commit kernel launch");
     i += k;
   }
@@ -196,43 +197,54 @@ APC_EXPORT apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t s
   return resolve(hp, step, out);
 }
 
-APC_EXPORT apc_status apc_commit_step_ex(const apc_tensor *table, int32_t num_tensors,
-                                         const apc_adamw_hparams *hp, int64_t step, uint32_t flags,
-                                         apc_stream_t stream, uint64_t *out_digests) {
-  g_last_error[0] = 0;
+namespace {
+
+// One table entry in layout-neutral form.
+struct TableRow {
+  void *p, *m, *v;
+  const uint16_t *g;
+  uint16_t *w;  // null for the bf16 layout
+  uint64_t n, goff;
+};
+
+// Shared by both layouts: validation, scalar resolution, overlap check,
+// planning and launches.  nslots digests are zeroed and accumulated.
+apc_status commit_common(int layout, const std::vector<TableRow> &rows, const apc_adamw_hparams *hp, int64_t step,
+                         uint32_t flags, apc_stream_t stream, uint64_t *out_digests, int nslots) {
   if (flags & ~(uint32_t)APC_COMMIT_ZERO_GRAD) return fail(APC_EINVAL, "unknown flag bits 0x%x", flags);
   const bool zero_grad = (flags & APC_COMMIT_ZERO_GRAD) != 0;
-  if (num_tensors < 0) return fail(APC_EINVAL, "num_tensors %d < 0", num_tensors);
-  if (num_tensors > 0 && !table) return fail(APC_EINVAL, "table pointer is null");
   if (!out_digests) return fail(APC_EINVAL, "out_digests pointer is null");
   if ((uintptr_t)out_digests % 8) return fail(APC_EALIGN, "out_digests not 8-byte aligned");
   float h[8];
   apc_status st = resolve(hp, step, h);
   if (st != APC_OK) return st;
+  const uint64_t es = layout == apc::kLayoutF32 ? 4 : 2;  // bytes per state element
 
   std::vector<apc::CommitEntry> entries;
   std::vector<Range> ranges;
-  entries.reserve((size_t)num_tensors);
-  ranges.reserve((size_t)num_tensors * 5);
-  for (int32_t k = 0; k < num_tensors; ++k) {
-    const apc_tensor &t = table[k];
+  entries.reserve(rows.size());
+  ranges.reserve(rows.size() * 5);
+  for (size_t k = 0; k < rows.size(); ++k) {
+    const TableRow &t = rows[k];
     if (t.n == 0) continue;
-    if (!t.p || !t.m || !t.v || !t.g || !t.w) return fail(APC_EINVAL, "table[%d]: null buffer pointer", k);
-    if (t.n > (UINT64_MAX - t.global_offset)) return fail(APC_ERANGE, "table[%d]: global_offset + n overflows", k);
-    if (t.n > ((uint64_t)1 << 61)) return fail(APC_ERANGE, "table[%d]: n too large", k);
+    if (!t.p || !t.m || !t.v || !t.g || (layout == apc::kLayoutF32 && !t.w))
+      return fail(APC_EINVAL, "table[%zu]: null buffer pointer", k);
+    if (t.n > (UINT64_MAX - t.goff)) return fail(APC_ERANGE, "table[%zu]: global_offset + n overflows", k);
+    if (t.n > ((uint64_t)1 << 61)) return fail(APC_ERANGE, "table[%zu]: n too large", k);
     const uintptr_t p = (uintptr_t)t.p, m = (uintptr_t)t.m, v = (uintptr_t)t.v, g = (uintptr_t)t.g,
                     w = (uintptr_t)t.w;
-    if (p % 4 || m % 4 || v % 4) return fail(APC_EALIGN, "table[%d]: fp32 buffer not 4-byte aligned", k);
-    if (g % 2 || w % 2) return fail(APC_EALIGN, "table[%d]: bf16 buffer not 2-byte aligned", k);
-    ranges.push_back({p, p + 4 * t.n, true});
-    ranges.push_back({m, m + 4 * t.n, true});
-    ranges.push_back({v, v + 4 * t.n, true});
-    ranges.push_back({w, w + 2 * t.n, true});
+    if (p % es || m % es || v % es)
+      return fail(APC_EALIGN, "table[%zu]: state buffer not %u-byte aligned", k, (unsigned)es);
+    if (g % 2 || w % 2) return fail(APC_EALIGN, "table[%zu]: bf16 buffer not 2-byte aligned", k);
+    ranges.push_back({p, p + es * t.n, true});
+    ranges.push_back({m, m + es * t.n, true});
+    ranges.push_back({v, v + es * t.n, true});
+    if (t.w) ranges.push_back({w, w + 2 * t.n, true});
     ranges.push_back({g, g + 2 * t.n, zero_grad});
-    // first element at which all five buffers sit on a 16-byte boundary
+    // first element at which all buffers sit on a 16-byte boundary
     const uint64_t h0 = ((16 - g % 16) % 16) / 2;
-    const bool aligned = (p + 4 * h0) % 16 == 0 && (m + 4 * h0) % 16 == 0 && (v + 4 * h0) % 16 == 0 &&
-                         (w + 2 * h0) % 16 == 0;
+    const bool aligned = (p + es * h0) % 16 == 0 && (m + es * h0) % 16 == 0 && (v + es * h0) % 16 == 0 &&
+                         (!t.w || (w + 2 * h0) % 16 == 0);
     apc::CommitEntry e;
     e.p = t.p;
     e.m = t.m;
@@ -240,7 +252,7 @@ APC_EXPORT apc_status apc_commit_step_ex(const apc_tensor *table, int32_t num_te
     e.g = t.g;
     e.w = t.w;
     e.n = t.n;
-    e.key_base = (uint32_t)t.global_offset;
+    e.key_base = (uint32_t)t.goff;
     if (aligned) {
       const uint64_t head = std::min<uint64_t>(h0, t.n);
       const uint64_t body = (t.n - head) / apc::kVec * apc::kVec;
@@ -256,22 +268,52 @@ APC_EXPORT apc_status apc_commit_step_ex(const apc_tensor *table, int32_t num_te
   }
   if (overlaps(ranges)) return fail(APC_EINVAL, "table buffers overlap (a written range meets another range)");
 
-  int e = (int)cudaMemsetAsync(out_digests, 0, 4 * sizeof(uint64_t), (cudaStream_t)stream);
+  int e = (int)cudaMemsetAsync(out_digests, 0, (size_t)nslots * sizeof(uint64_t), (cudaStream_t)stream);
   if (e) return cuda_fail(e, "cudaMemsetAsync(out_digests)");
   if (entries.empty()) return APC_OK;
   Device d;
   if ((st = device_info(&d)) != APC_OK) return st;
   unsigned long long *out = reinterpret_cast<unsigned long long *>(out_digests);
   if (entries.size() <= (size_t)apc::kCommitSmall)
-    return run_commit_batches<apc::kCommitSmall>(entries, h, zero_grad, grid_for(UINT64_MAX, d.sms, d.commit_small),
-                                                 stream, out, apc::launch_commit_small);
-  return run_commit_batches<apc::kCommitLarge>(entries, h, zero_grad, grid_for(UINT64_MAX, d.sms, d.commit_large),
-                                               stream, out, apc::launch_commit_large);
+    return run_commit_batches<apc::kCommitSmall>(entries, h, layout, zero_grad,
+                                                 grid_for(UINT64_MAX, d.sms, d.commit_small), stream, out,
+                                                 apc::launch_commit_small);
+  return run_commit_batches<apc::kCommitLarge>(entries, h, layout, zero_grad,
+                                               grid_for(UINT64_MAX, d.sms, d.commit_large), stream, out,
+                                               apc::launch_commit_large);
+}
+
+}  // namespace
+
+APC_EXPORT apc_status apc_commit_step_ex(const apc_tensor *table, int32_t num_tensors,
+                                         const apc_adamw_hparams *hp, int64_t step, uint32_t flags,
+                                         apc_stream_t stream, uint64_t *out_digests) {
+  g_last_error[0] = 0;
+  if (num_tensors < 0) return fail(APC_EINVAL, "num_tensors %d < 0", num_tensors);
+  if (num_tensors > 0 && !table) return fail(APC_EINVAL, "table pointer is null");
+  std::vector<TableRow> rows((size_t)num_tensors);
+  for (int32_t k = 0; k < num_tensors; ++k)
+    rows[k] = TableRow{table[k].p, table[k].m, table[k].v, table[k].g, table[k].w, table[k].n,
+                       table[k].global_offset};
+  return commit_common(apc::kLayoutF32, rows, hp, step, flags, stream, out_digests, 4);
 }
 
 APC_EXPORT apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
                                       int64_t step, apc_stream_t stream, uint64_t *out_digests) {
   return apc_commit_step_ex(table, num_tensors, hp, step, 0u, stream, out_digests);
+}
+
+APC_EXPORT apc_status apc_commit_step_bf16(const apc_tensor_bf16 *table, int32_t num_tensors,
+                                           const apc_adamw_hparams *hp, int64_t step, uint32_t flags,
+                                           apc_stream_t stream, uint64_t *out_digests) {
+  g_last_error[0] = 0;
+  if (num_tensors < 0) return fail(APC_EINVAL, "num_tensors %d < 0", num_tensors);
+  if (num_tensors > 0 && !table) return fail(APC_EINVAL, "table pointer is null");
+  std::vector<TableRow> rows((size_t)num_tensors);
+  for (int32_t k = 0; k < num_tensors; ++k)
+    rows[k] = TableRow{table[k].p, table[k].m, table[k].v, table[k].g, nullptr, table[k].n,
+                       table[k].global_offset};
+  return commit_common(apc::kLayoutBF16, rows, hp, step, flags, stream, out_digests, 3);
 }
 
 namespace {

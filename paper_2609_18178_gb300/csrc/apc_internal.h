@@ -45,16 +45,22 @@ constexpr uint32_t kCommitSmemBytes = kCommitStages * kCommitStageBytes;
 constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
 static_assert(kCommitSmemBytes <= 227 * 1024, "shared memory per CTA");
 
+// State layouts of the commit kernel.
+constexpr int kLayoutF32 = 0;   // fp32 p, m, v; bf16 g; bf16 copy w
+constexpr int kLayoutBF16 = 1;  // bf16 p, m, v; bf16 g; no copy
+
 // One chunk-table entry of the commit kernel (72 bytes).
+//   p, m, v: fp32 or bf16 state (by the launch's layout); w: the bf16 copy
+//         (fp32 layout only).
 //   head: elements [0, head) are scalar items, then 16-byte aligned vectors
 //         up to vec_end = head + 8 * floor((n - head) / 8) in tiles of
-//         kCommitTile, then scalar items up to n; kScalarMode when the five
+//         kCommitTile, then scalar items up to n; kScalarMode when the
 //         buffers are not mutually 16-byte aligned (all n elements scalar).
 //   tile_begin: the entry's first tile in the launch's tile space.
 //   scalar_begin: the entry's first item in the launch's scalar-item space.
 //   key_base: global_offset mod 2^32 (the digest key of element 0).
 struct CommitEntry {
-  float *p, *m, *v;
+  void *p, *m, *v;
   const uint16_t *g;
   uint16_t *w;
   uint64_t n;
@@ -116,10 +122,10 @@ static_assert(sizeof(DigestPlan<kDigestLarge>) <= 32764, "kernel parameter limit
 
 // Launch wrappers (apc_commit.cu, apc_digest.cu).  They return a cudaError_t
 // value and launch on `stream` with `grid` CTAs.
-int launch_commit_small(const CommitPlan<kCommitSmall> &plan, bool zero_grad, unsigned grid, void *stream,
-                        unsigned long long *out);
-int launch_commit_large(const CommitPlan<kCommitLarge> &plan, bool zero_grad, unsigned grid, void *stream,
-                        unsigned long long *out);
+int launch_commit_small(const CommitPlan<kCommitSmall> &plan, int layout, bool zero_grad, unsigned grid,
+                        void *stream, unsigned long long *out);
+int launch_commit_large(const CommitPlan<kCommitLarge> &plan, int layout, bool zero_grad, unsigned grid,
+                        void *stream, unsigned long long *out);
 int launch_digest_small(const DigestPlan<kDigestSmall> &plan, unsigned grid, void *stream,
                         unsigned long long *out);
 int launch_digest_large(const DigestPlan<kDigestLarge> &plan, unsigned grid, void *stream,

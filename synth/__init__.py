@@ -20,6 +20,7 @@ import numpy as np
 
 P, M, V, G = 1, 2, 3, 4
 GZERO = 5
+P16, M16, V16 = 6, 7, 8
 SEED = 0
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -100,7 +101,7 @@ def _dev_lib():
 def _dtype(kind: int):
     if kind in (P, M, V):
         return np.float32
-    if kind == G:
+    if kind in (G, P16, M16, V16):
         return np.uint16
     raise ValueError("unknown synthetic buffer kind %r" % (kind,))
 
@@ -157,6 +158,12 @@ def state(n: int, goff: int = 0, seed: int = SEED, nthreads: int | None = None):
     """(p, m, v) fp32 state arrays of one contiguous global range."""
     return (fill(P, n, goff, 0, seed, nthreads), fill(M, n, goff, 0, seed, nthreads),
             fill(V, n, goff, 0, seed, nthreads))
+
+
+def state_bf16(n: int, goff: int = 0, seed: int = SEED, nthreads: int | None = None):
+    """(p, m, v) bf16 state bits (uint16) of one contiguous global range."""
+    return (fill(P16, n, goff, 0, seed, nthreads), fill(M16, n, goff, 0, seed, nthreads),
+            fill(V16, n, goff, 0, seed, nthreads))
 
 
 def grad(n: int, goff: int = 0, step: int = 1, seed: int = SEED, nthreads: int | None = None):

@@ -25,6 +25,7 @@
  *   g  = top 16 bits of fp32(1e-3 * z)   bf16 gradient ~ N(0, 1e-3), made by
  *        truncation; exactly +0 when word 0 of call 0 of kind GZERO is a
  *        multiple of 100 (1% exact zeros).  The gradient depends on the step.
+ *   p16, m16, v16 = top 16 bits of p, m, v  (bf16 state, by truncation)
  * Only integer operations and single IEEE-rounded double/float operations are
  * used, so host and device produce the same bits.
  */
@@ -44,7 +45,10 @@ enum {
   SYNTH_M = 2,      /* fp32 first moment                 */
   SYNTH_V = 3,      /* fp32 second moment                */
   SYNTH_G = 4,      /* bf16 gradient (depends on step)   */
-  SYNTH_GZERO = 5   /* zero mask of the gradient         */
+  SYNTH_GZERO = 5,  /* zero mask of the gradient         */
+  SYNTH_P16 = 6,    /* bf16 parameters: top half of SYNTH_P's value */
+  SYNTH_M16 = 7,    /* bf16 first moment: top half of SYNTH_M's     */
+  SYNTH_V16 = 8     /* bf16 second moment: top half of SYNTH_V's    */
 };
 
 SYNTH_HD void synth_mulhilo(uint32_t a, uint32_t b, uint32_t *hi, uint32_t *lo) {
@@ -119,5 +123,9 @@ SYNTH_HD uint16_t synth_g(uint64_t seed, uint64_t i, int64_t step) {
   float x = (float)(1e-3 * synth_normal(seed, SYNTH_G, i, step));
   return (uint16_t)(synth_f32_bits(x) >> 16);
 }
+
+SYNTH_HD uint16_t synth_p16(uint64_t seed, uint64_t i) { return (uint16_t)(synth_f32_bits(synth_p(seed, i)) >> 16); }
+SYNTH_HD uint16_t synth_m16(uint64_t seed, uint64_t i) { return (uint16_t)(synth_f32_bits(synth_m(seed, i)) >> 16); }
+SYNTH_HD uint16_t synth_v16(uint64_t seed, uint64_t i) { return (uint16_t)(synth_f32_bits(synth_v(seed, i)) >> 16); }
 
 #endif /* SYNTH_PHILOX_H */

@@ -24,6 +24,9 @@ __global__ void synth_fill_kernel(int kind, uint64_t seed, uint64_t goff, uint64
       case SYNTH_M: f[j] = synth_m(seed, i); break;
       case SYNTH_V: f[j] = synth_v(seed, i); break;
       case SYNTH_G: h[j] = synth_g(seed, i, step); break;
+      case SYNTH_P16: h[j] = synth_p16(seed, i); break;
+      case SYNTH_M16: h[j] = synth_m16(seed, i); break;
+      case SYNTH_V16: h[j] = synth_v16(seed, i); break;
       default: break;
     }
   }
@@ -34,7 +37,7 @@ __global__ void synth_fill_kernel(int kind, uint64_t seed, uint64_t goff, uint64
  * Returns a cudaError_t value (0 on success); -1 on a bad kind. */
 SYNTH_EXPORT int synth_fill_dev(int kind, uint64_t seed, uint64_t goff, uint64_t n, int64_t step,
                                 void *out, void *stream) {
-  if (kind < SYNTH_P || kind > SYNTH_G) return -1;
+  if (kind < SYNTH_P || kind > SYNTH_V16 || kind == SYNTH_GZERO) return -1;
   if (n == 0) return 0;
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);

@@ -24,6 +24,9 @@ static void fill_range(int kind, uint64_t seed, uint64_t goff, uint64_t lo, uint
       case SYNTH_M: f[j] = synth_m(seed, i); break;
       case SYNTH_V: f[j] = synth_v(seed, i); break;
       case SYNTH_G: h[j] = synth_g(seed, i, step); break;
+      case SYNTH_P16: h[j] = synth_p16(seed, i); break;
+      case SYNTH_M16: h[j] = synth_m16(seed, i); break;
+      case SYNTH_V16: h[j] = synth_v16(seed, i); break;
       default: break;
     }
   }
@@ -43,11 +46,11 @@ static void *fill_worker(void *arg) {
 }
 
 /* Fill out[0..n) with the values of global indices goff..goff+n-1.
- * kind: SYNTH_P/M/V (float out) or SYNTH_G (uint16 bf16 bits out).
+ * kind: SYNTH_P/M/V (float out) or SYNTH_G/P16/M16/V16 (uint16 bf16 bits out).
  * Returns 0 on success, -1 on a bad kind. */
 SYNTH_EXPORT int synth_fill(int kind, uint64_t seed, uint64_t goff, uint64_t n, int64_t step,
                             void *out, int nthreads) {
-  if (kind < SYNTH_P || kind > SYNTH_G) return -1;
+  if (kind < SYNTH_P || kind > SYNTH_V16 || kind == SYNTH_GZERO) return -1;
   if (nthreads < 1) nthreads = 1;
   if (nthreads > 256) nthreads = 256;
   if ((uint64_t)nthreads > n / 65536 + 1) nthreads = (int)(n / 65536 + 1);
@@ -74,7 +77,7 @@ SYNTH_EXPORT int synth_fill(int kind, uint64_t seed, uint64_t goff, uint64_t n, 
 /* Values at arbitrary global indices idx[0..n). */
 SYNTH_EXPORT int synth_fill_at(int kind, uint64_t seed, const uint64_t *idx, uint64_t n, int64_t step,
                                void *out) {
-  if (kind < SYNTH_P || kind > SYNTH_G) return -1;
+  if (kind < SYNTH_P || kind > SYNTH_V16 || kind == SYNTH_GZERO) return -1;
   float *f = (float *)out;
   uint16_t *h = (uint16_t *)out;
   for (uint64_t j = 0; j < n; ++j) {
@@ -83,6 +86,9 @@ SYNTH_EXPORT int synth_fill_at(int kind, uint64_t seed, const uint64_t *idx, uin
       case SYNTH_M: f[j] = synth_m(seed, idx[j]); break;
       case SYNTH_V: f[j] = synth_v(seed, idx[j]); break;
       case SYNTH_G: h[j] = synth_g(seed, idx[j], step); break;
+      case SYNTH_P16: h[j] = synth_p16(seed, idx[j]); break;
+      case SYNTH_M16: h[j] = synth_m16(seed, idx[j]); break;
+      case SYNTH_V16: h[j] = synth_v16(seed, idx[j]); break;
       default: break;
     }
   }

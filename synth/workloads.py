@@ -19,6 +19,7 @@ Workloads:
       step 5, then a verification digest.
   c5  the full Mistral-7B model, 291 separately allocated tensors; step 18,
       then a verification digest.
+  f3  bf16-state rank shard of the 4-way sharded Mistral-7B (rank 1 of 4).
 """
 from __future__ import annotations
 
@@ -138,6 +139,16 @@ def c4(rank: int = 9, world: int = 16, one_entry: bool = False) -> Workload:
 def c5() -> Workload:
     pieces, allocs = _separate(mistral_tensors())
     return Workload("c5", pieces, [18], chained=False, verify=True, allocs=allocs)
+
+
+def f3(rank: int = 1, world: int = 4) -> Workload:
+    """The paper's own per-rank shard: Mistral-7B under 4-way intra-node
+    sharding (Section IV-A; 10.9 GB of BF16 state per rank, Section II-B),
+    rank 1 of 4 = 1,812,005,888 elements across tensor boundaries, one flat
+    allocation, bf16 state; step 5, then a verification digest."""
+    w = c4(rank, world)
+    w.name, w.steps = "f3", [5]
+    return w
 
 
 ALL = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5}

@@ -147,3 +147,83 @@ def sample_indices(w: W.Workload, k: int, seed: int) -> np.ndarray:
     j = np.searchsorted(starts, r, side="right") - 1
     idx += [w.pieces[a].goff + int(r[i] - starts[a]) for i, a in enumerate(j)]
     return np.unique(np.array(idx, dtype=np.uint64))
+
+
+class DeviceWorkloadBF16:
+    """bf16 p, m, v and g per allocation of a workload on the current CUDA
+    device, filled from the generator by the device fill."""
+
+    def __init__(self, w: W.Workload, grad_step: int, device="cuda"):
+        import torch
+        self.w = w
+        self.alloc_goff = [None] * len(w.allocs)
+        for p in w.pieces:
+            self.alloc_goff[p.alloc] = p.goff - p.at
+        s = torch.cuda.current_stream().cuda_stream
+        self.bufs = []
+        for a, n in enumerate(w.allocs):
+            b = {k: torch.empty(n, dtype=torch.int16, device=device) for k in "pmvg"}
+            g0 = self.alloc_goff[a]
+            synth.fill_dev(synth.P16, b["p"].data_ptr(), n, g0, stream=s)
+            synth.fill_dev(synth.M16, b["m"].data_ptr(), n, g0, stream=s)
+            synth.fill_dev(synth.V16, b["v"].data_ptr(), n, g0, stream=s)
+            synth.fill_dev(synth.G, b["g"].data_ptr(), n, g0, step=grad_step, stream=s)
+            self.bufs.append(b)
+
+    def entries(self):
+        import paper_2609_18178_gb300 as apc
+        out = []
+        for p in self.w.pieces:
+            b = self.bufs[p.alloc]
+            sl = slice(p.at, p.at + p.n)
+            out.append(apc.TensorEntryBF16(b["p"][sl], b["m"][sl], b["v"][sl], b["g"][sl], p.goff))
+        return out
+
+    def digest_buffers(self):
+        import paper_2609_18178_gb300 as apc
+        out = []
+        for p in self.w.pieces:
+            b = self.bufs[p.alloc]
+            sl = slice(p.at, p.at + p.n)
+            out += apc.state_buffers_bf16(b["p"][sl], b["m"][sl], b["v"][sl], p.goff)
+        return out
+
+    def gather(self, gidx: np.ndarray):
+        import torch
+        starts = np.array([p.goff for p in self.w.pieces], dtype=np.int64)
+        k = np.searchsorted(starts, gidx.astype(np.int64), side="right") - 1
+        alloc = np.array([self.w.pieces[i].alloc for i in k])
+        off = gidx.astype(np.int64) - starts[k] + np.array([self.w.pieces[i].at for i in k])
+        res = {key: np.empty(len(gidx), dtype=np.uint16) for key in "pmv"}
+        for a in np.unique(alloc):
+            sel = np.nonzero(alloc == a)[0]
+            idx = torch.from_numpy(off[sel]).to(self.bufs[a]["p"].device)
+            for key in "pmv":
+                res[key][sel] = self.bufs[a][key].index_select(0, idx).cpu().numpy().view(np.uint16)
+        return res
+
+
+def oracle_at_bf16(gidx: np.ndarray, step: int, hp=None):
+    """Oracle outputs of one bf16-state step from the generated state at global indices."""
+    hp = hp or oracle.DEFAULT_HP
+    p = synth.fill_at(synth.P16, gidx)
+    m = synth.fill_at(synth.M16, gidx)
+    v = synth.fill_at(synth.V16, gidx)
+    g = synth.fill_at(synth.G, gidx, step=step)
+    oracle.adamw_bf16(p, m, v, g, oracle.resolve_hparams(hp, step))
+    return dict(p=p, m=m, v=v)
+
+
+def oracle_workload_digest_bf16(w: W.Workload, step: int, lo: int, hi: int, hp=None, chunk: int = 1 << 24):
+    """The three bf16-state digests of one step over the part [lo, hi) of a
+    workload's global range, streamed through the oracle."""
+    hp = hp or oracle.DEFAULT_HP
+    h8 = oracle.resolve_hparams(hp, step)
+    tot = [0, 0, 0]
+    for s in range(lo, hi, chunk):
+        n = min(chunk, hi - s)
+        p, m, v = synth.state_bf16(n, s, nthreads=NTHREADS)
+        g = synth.grad(n, s, step, nthreads=NTHREADS)
+        d = oracle.commit_bf16(p, m, v, g, s, h8)
+        tot = [(a + b) & M64 for a, b in zip(tot, d)]
+    return tot

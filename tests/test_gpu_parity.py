@@ -432,3 +432,98 @@ def test_count_nonzero_of_arbitrary_buffers():
         keep.append(t)
         bufs.append(apc.BufferEntry(t[shift:], slot, 0, apc.F32 if f32 else apc.BF16))
     assert apc.digests_to_host(apc.count_nonzero(bufs, 8)) == want
+
+
+# --------------------------------------------------------- bf16 state (f3)
+
+from apc_testlib import DeviceWorkloadBF16, oracle_at_bf16, oracle_workload_digest_bf16  # noqa: E402
+
+
+def gen16(n, goff, step):
+    p, m, v = synth.state_bf16(n, goff)
+    return dict(p=p, m=m, v=v, g=synth.grad(n, goff, step), goff=goff)
+
+
+def run_bf16(tensors, step, hp=HP, zero_grad=False, shift=0):
+    """Commit bf16-state tensors (each optionally viewed `shift` elements
+    into its buffers) and compare every word and digest with the oracle."""
+    devs, entries = [], []
+    for t in tensors:
+        n = t["p"].size
+        d = {k: dev(np.concatenate([np.zeros(shift, np.uint16), t[k]])) for k in "pmvg"}
+        devs.append(d)
+        sl = slice(shift, shift + n)
+        entries.append(apc.TensorEntryBF16(d["p"][sl], d["m"][sl], d["v"][sl], d["g"][sl], t["goff"]))
+    out = apc.commit_step_bf16(entries, step, hp, zero_grad=zero_grad)
+    torch.cuda.synchronize()
+    h8 = oracle.resolve_hparams(hp, step)
+    want = [0, 0, 0]
+    for t, d in zip(tensors, devs):
+        p, m, v = t["p"].copy(), t["m"].copy(), t["v"].copy()
+        dd = oracle.commit_bf16(p, m, v, t["g"], t["goff"], h8)
+        want = [(a + b) & M64 for a, b in zip(want, dd)]
+        sl = slice(shift, shift + p.size)
+        for k, ref in (("p", p), ("m", m), ("v", v)):
+            assert np.array_equal(host(d[k], np.uint16)[sl], ref), k
+        g_after = host(d["g"], np.uint16)[sl]
+        assert (not g_after.any()) if zero_grad else np.array_equal(g_after, t["g"])
+    assert apc.digests_to_host(out) == want
+
+
+@pytest.mark.parametrize("n", [1, 3, 7, 8, 9, 63, 4864, 4871, 9728 + 5, 100003])
+def test_bf16_state_sizes(n):
+    run_bf16([gen16(n, (1 << 32) - n // 3, 2)], 2)
+
+
+@pytest.mark.parametrize("shift", [1, 3, 5, 7])
+def test_bf16_state_misaligned_views(shift):
+    run_bf16([gen16(20000, 77, 3), gen16(513, 20077, 3)], 3, shift=shift)
+
+
+def test_bf16_state_mutual_misalignment_runs_scalar():
+    n = 5000
+    t = gen16(n + 8, 0, 4)
+    d = {k: dev(t[k]) for k in "pmvg"}
+    e = apc.TensorEntryBF16(d["p"][1:n + 1], d["m"][1:n + 1], d["v"][1:n + 1], d["g"][0:n], 9)
+    out = apc.commit_step_bf16([e], 4, HP)
+    torch.cuda.synchronize()
+    p, m, v = t["p"][1:n + 1].copy(), t["m"][1:n + 1].copy(), t["v"][1:n + 1].copy()
+    want = oracle.commit_bf16(p, m, v, np.ascontiguousarray(t["g"][0:n]), 9, oracle.resolve_hparams(HP, 4))
+    assert np.array_equal(host(d["p"], np.uint16)[1:n + 1], p)
+    assert np.array_equal(host(d["v"], np.uint16)[1:n + 1], v)
+    assert apc.digests_to_host(out) == want
+
+
+def test_bf16_state_many_tensors_zero_grad_and_hparams():
+    rng = np.random.default_rng(41)
+    tensors, off = [], 12345
+    for n in rng.integers(1, 2000, size=500):
+        tensors.append(gen16(int(n), off, 6))
+        off += int(n)
+    run_bf16(tensors, 6, zero_grad=True)
+    run_bf16(tensors[:40], 1000, dict(lr=1e-2, beta1=0.0, beta2=0.999, eps=1e-6, weight_decay=0.0))
+
+
+def test_f3_rank_shard_bf16_full_size():
+    """The paper's 4-way rank shard of Mistral-7B in bf16 state (1,812,005,888
+    elements, 77 pieces of one allocation): sampled words against the
+    oracle, the verification digest equals the fused one, and the digests of
+    a 64 Mi-element slice equal the streamed oracle's."""
+    w = W.f3()
+    dw = DeviceWorkloadBF16(w, 5)
+    got = apc.digests_to_host(apc.commit_step_bf16(dw.entries(), 5, HP))
+    idx = sample_indices(w, 200000, 7)
+    res = dw.gather(idx)
+    ref = oracle_at_bf16(idx, 5)
+    for k in "pmv":
+        assert np.array_equal(res[k], ref[k]), k
+    assert apc.digests_to_host(apc.digest(dw.digest_buffers(), 3)) == got
+    lo = w.pieces[0].goff + 123_456_789
+    hi = lo + (64 << 20)
+    start = lo - (w.pieces[0].goff - w.pieces[0].at)
+    b = dw.bufs[0]
+    sl = slice(start, start + (hi - lo))
+    part = apc.digests_to_host(apc.digest(apc.state_buffers_bf16(b["p"][sl], b["m"][sl], b["v"][sl], lo), 3))
+    assert part == oracle_workload_digest_bf16(w, 5, lo, hi)
+    del dw
+    torch.cuda.empty_cache()
