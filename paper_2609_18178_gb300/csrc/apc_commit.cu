@@ -95,14 +95,22 @@ struct F32State {
     __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.m) + i), make_float4(m[0], m[1], m[2], m[3]));
     __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.v) + i), make_float4(v[0], v[1], v[2], v[3]));
     __stcs(reinterpret_cast<uint2 *>(E.w + i), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
-    a.p += digest_term(G, __float_as_uint(p[0])) + digest_term(G + 1, __float_as_uint(p[1]));
-    a.p += digest_term(G + 2, __float_as_uint(p[2])) + digest_term(G + 3, __float_as_uint(p[3]));
-    a.m += digest_term(G, __float_as_uint(m[0])) + digest_term(G + 1, __float_as_uint(m[1]));
-    a.m += digest_term(G + 2, __float_as_uint(m[2])) + digest_term(G + 3, __float_as_uint(m[3]));
-    a.v += digest_term(G, __float_as_uint(v[0])) + digest_term(G + 1, __float_as_uint(v[1]));
-    a.v += digest_term(G + 2, __float_as_uint(v[2])) + digest_term(G + 3, __float_as_uint(v[3]));
-    a.w += digest_term(G, w[0]) + digest_term(G + 1, w[1]);
-    a.w += digest_term(G + 2, w[2]) + digest_term(G + 3, w[3]);
+    acc_add(a.p, digest_term(G, __float_as_uint(p[0]), s.one), s.one);
+    acc_add(a.p, digest_term(G + 1, __float_as_uint(p[1]), s.one), s.one);
+    acc_add(a.p, digest_term(G + 2, __float_as_uint(p[2]), s.one), s.one);
+    acc_add(a.p, digest_term(G + 3, __float_as_uint(p[3]), s.one), s.one);
+    acc_add(a.m, digest_term(G, __float_as_uint(m[0]), s.one), s.one);
+    acc_add(a.m, digest_term(G + 1, __float_as_uint(m[1]), s.one), s.one);
+    acc_add(a.m, digest_term(G + 2, __float_as_uint(m[2]), s.one), s.one);
+    acc_add(a.m, digest_term(G + 3, __float_as_uint(m[3]), s.one), s.one);
+    acc_add(a.v, digest_term(G, __float_as_uint(v[0]), s.one), s.one);
+    acc_add(a.v, digest_term(G + 1, __float_as_uint(v[1]), s.one), s.one);
+    acc_add(a.v, digest_term(G + 2, __float_as_uint(v[2]), s.one), s.one);
+    acc_add(a.v, digest_term(G + 3, __float_as_uint(v[3]), s.one), s.one);
+    acc_add(a.w, digest_term(G, w[0], s.one), s.one);
+    acc_add(a.w, digest_term(G + 1, w[1], s.one), s.one);
+    acc_add(a.w, digest_term(G + 2, w[2], s.one), s.one);
+    acc_add(a.w, digest_term(G + 3, w[3], s.one), s.one);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -114,10 +122,10 @@ struct F32State {
     V[i] = v;
     E.w[i] = (uint16_t)w;
     const uint32_t G = E.key_base + (uint32_t)i;
-    a.p += digest_term(G, __float_as_uint(p));
-    a.m += digest_term(G, __float_as_uint(m));
-    a.v += digest_term(G, __float_as_uint(v));
-    a.w += digest_term(G, w);
+    acc_add(a.p, digest_term(G, __float_as_uint(p), s.one), s.one);
+    acc_add(a.m, digest_term(G, __float_as_uint(m), s.one), s.one);
+    acc_add(a.v, digest_term(G, __float_as_uint(v), s.one), s.one);
+    acc_add(a.w, digest_term(G, w, s.one), s.one);
   }
 };
 
@@ -157,12 +165,18 @@ struct BF16State {
            make_uint2(mo[0] | (mo[1] << 16), mo[2] | (mo[3] << 16)));
     __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(E.v) + i),
            make_uint2(vo[0] | (vo[1] << 16), vo[2] | (vo[3] << 16)));
-    a.p += digest_term(G, po[0]) + digest_term(G + 1, po[1]);
-    a.p += digest_term(G + 2, po[2]) + digest_term(G + 3, po[3]);
-    a.m += digest_term(G, mo[0]) + digest_term(G + 1, mo[1]);
-    a.m += digest_term(G + 2, mo[2]) + digest_term(G + 3, mo[3]);
-    a.v += digest_term(G, vo[0]) + digest_term(G + 1, vo[1]);
-    a.v += digest_term(G + 2, vo[2]) + digest_term(G + 3, vo[3]);
+    acc_add(a.p, digest_term(G, po[0], s.one), s.one);
+    acc_add(a.p, digest_term(G + 1, po[1], s.one), s.one);
+    acc_add(a.p, digest_term(G + 2, po[2], s.one), s.one);
+    acc_add(a.p, digest_term(G + 3, po[3], s.one), s.one);
+    acc_add(a.m, digest_term(G, mo[0], s.one), s.one);
+    acc_add(a.m, digest_term(G + 1, mo[1], s.one), s.one);
+    acc_add(a.m, digest_term(G + 2, mo[2], s.one), s.one);
+    acc_add(a.m, digest_term(G + 3, mo[3], s.one), s.one);
+    acc_add(a.v, digest_term(G, vo[0], s.one), s.one);
+    acc_add(a.v, digest_term(G + 1, vo[1], s.one), s.one);
+    acc_add(a.v, digest_term(G + 2, vo[2], s.one), s.one);
+    acc_add(a.v, digest_term(G + 3, vo[3], s.one), s.one);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -174,9 +188,9 @@ struct BF16State {
     M[i] = (uint16_t)mo;
     V[i] = (uint16_t)vo;
     const uint32_t G = E.key_base + (uint32_t)i;
-    a.p += digest_term(G, po);
-    a.m += digest_term(G, mo);
-    a.v += digest_term(G, vo);
+    acc_add(a.p, digest_term(G, po, s.one), s.one);
+    acc_add(a.m, digest_term(G, mo, s.one), s.one);
+    acc_add(a.v, digest_term(G, vo, s.one), s.one);
   }
 };
 
@@ -265,7 +279,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
     __syncwarp();
   } else {
     // ----------------------------------------------------------- consumers
-    const Scalars s{plan.h};
+    const Scalars s{plan.h, plan.one};
     const int ct = threadIdx.x;  // 0 .. kCommitConsumers-1
     uint32_t cur = 0, phase = 0;
     int stage = 0;

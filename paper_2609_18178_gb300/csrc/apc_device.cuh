@@ -20,6 +20,7 @@ namespace apc {
 // every use is a constant-bank operand and holds no register.
 struct Scalars {
   const float *h;  // b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/(1-b1^t), 1/sqrt(1-b2^t)
+  uint32_t one;    // 1, from the launch parameters (see digest_term)
 };
 
 // One element: p, m, v updated in place, returns the bf16 bits of p'.
@@ -48,11 +49,32 @@ __device__ __forceinline__ uint32_t adamw_element(float &p, float &m, float &v, 
 // splitmix64 of the digest key ((G mod 2^32) << 32) | bits: the first output
 // of Vigna's SplitMix64 seeded with the key (golden-ratio increment, then the
 // 30/27/31 xor-shift multiply finaliser).
-__device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits) {
-  uint64_t z = (((uint64_t)gidx << 32) | bits) + 0x9E3779B97F4A7C15ull;
+//
+// Instruction mix: the kernels are short of integer-ALU issue, so the 64-bit
+// increment puts its high half on the FMA pipe as an extended-precision
+// multiply-add by `one` (a launch parameter equal to 1, so the assembler
+// cannot turn it back into an ALU add): lo = bits + 0x7F4A7C15 sets the
+// carry, hi = G * one + 0x9E3779B9 + carry.
+__device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits, uint32_t one) {
+  uint32_t lo, hi;
+  asm("add.cc.u32 %0, %2, 0x7F4A7C15;\n\t"
+      "madc.lo.u32 %1, %3, %4, 0x9E3779B9;"
+      : "=r"(lo), "=r"(hi)
+      : "r"(bits), "r"(gidx), "r"(one));
+  uint64_t z = ((uint64_t)hi << 32) | lo;
   z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
   z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
   return z ^ (z >> 31);
+}
+
+// acc += z (mod 2^64), with the high half's carry-add on the FMA pipe.
+__device__ __forceinline__ void acc_add(uint64_t &acc, uint64_t z, uint32_t one) {
+  uint32_t alo = (uint32_t)acc, ahi = (uint32_t)(acc >> 32);
+  asm("add.cc.u32 %0, %0, %2;\n\t"
+      "madc.lo.u32 %1, %3, %4, %1;"
+      : "+r"(alo), "+r"(ahi)
+      : "r"((uint32_t)z), "r"((uint32_t)(z >> 32)), "r"(one));
+  acc = ((uint64_t)ahi << 32) | alo;
 }
 
 // Sum of a CTA's per-thread values; the result is valid in thread 0.

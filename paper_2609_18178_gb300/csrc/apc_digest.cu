@@ -42,6 +42,7 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
   __shared__ unsigned long long s_acc[APC_MAX_SLOTS];
   if (threadIdx.x < APC_MAX_SLOTS) s_acc[threadIdx.x] = 0;
   __syncthreads();
+  const uint32_t one = plan.one;
   uint32_t cur = 0;
   int slot = -1;
   uint64_t acc = 0;
@@ -74,10 +75,14 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
       for (int u = 0; u < kDigestUnroll; ++u) {
         if (!ok[u]) continue;
         const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        t0 += digest_term(G + 0, x[u][0].x) + digest_term(G + 1, x[u][0].y);
-        t1 += digest_term(G + 2, x[u][0].z) + digest_term(G + 3, x[u][0].w);
-        t0 += digest_term(G + 4, x[u][1].x) + digest_term(G + 5, x[u][1].y);
-        t1 += digest_term(G + 6, x[u][1].z) + digest_term(G + 7, x[u][1].w);
+        acc_add(t0, digest_term(G + 0, x[u][0].x, one), one);
+        acc_add(t0, digest_term(G + 1, x[u][0].y, one), one);
+        acc_add(t1, digest_term(G + 2, x[u][0].z, one), one);
+        acc_add(t1, digest_term(G + 3, x[u][0].w, one), one);
+        acc_add(t0, digest_term(G + 4, x[u][1].x, one), one);
+        acc_add(t0, digest_term(G + 5, x[u][1].y, one), one);
+        acc_add(t1, digest_term(G + 6, x[u][1].z, one), one);
+        acc_add(t1, digest_term(G + 7, x[u][1].w, one), one);
       }
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
@@ -93,21 +98,26 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
       for (int u = 0; u < kDigestUnroll; ++u) {
         if (!ok[u]) continue;
         const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        t0 += digest_term(G + 0, x[u].x & 0xFFFFu) + digest_term(G + 1, x[u].x >> 16);
-        t1 += digest_term(G + 2, x[u].y & 0xFFFFu) + digest_term(G + 3, x[u].y >> 16);
-        t0 += digest_term(G + 4, x[u].z & 0xFFFFu) + digest_term(G + 5, x[u].z >> 16);
-        t1 += digest_term(G + 6, x[u].w & 0xFFFFu) + digest_term(G + 7, x[u].w >> 16);
+        acc_add(t0, digest_term(G + 0, x[u].x & 0xFFFFu, one), one);
+        acc_add(t0, digest_term(G + 1, x[u].x >> 16, one), one);
+        acc_add(t1, digest_term(G + 2, x[u].y & 0xFFFFu, one), one);
+        acc_add(t1, digest_term(G + 3, x[u].y >> 16, one), one);
+        acc_add(t0, digest_term(G + 4, x[u].z & 0xFFFFu, one), one);
+        acc_add(t0, digest_term(G + 5, x[u].z >> 16, one), one);
+        acc_add(t1, digest_term(G + 6, x[u].w & 0xFFFFu, one), one);
+        acc_add(t1, digest_term(G + 7, x[u].w >> 16, one), one);
       }
     }
     if (local == 0) {
       const uint32_t t = threadIdx.x;
-      if (t < head) t0 += digest_term(E.key_base + t, word_at(E, t));
+      if (t < head) { acc_add(t0, digest_term(E.key_base + t, word_at(E, t), one), one); }
       if (t >= 32 && t - 32 < E.n - vec_end) {
         const uint64_t i = vec_end + (t - 32);
-        t0 += digest_term(E.key_base + (uint32_t)i, word_at(E, i));
+        acc_add(t0, digest_term(E.key_base + (uint32_t)i, word_at(E, i), one), one);
       }
     }
-    acc += t0 + t1;
+    acc_add(acc, t0, one);
+    acc_add(acc, t1, one);
   }
   flush(acc, slot, s_acc);
   __syncthreads();

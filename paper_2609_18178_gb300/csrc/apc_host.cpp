@@ -137,6 +137,7 @@ apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, cons
                               Launch launch) {
   auto plan = std::make_unique<apc::CommitPlan<MAXE>>();
   std::memcpy(plan->h, h, sizeof plan->h);
+  plan->one = 1;
   size_t i = 0;
   while (i < entries.size()) {
     const size_t k = std::min(entries.size() - i, (size_t)MAXE);
@@ -166,6 +167,7 @@ template <int MAXE, typename Launch>
 apc_status run_digest_batches(const std::vector<apc::DigestEntry> &entries, unsigned grid_cap, void *stream,
                               unsigned long long *out, Launch launch, const char *what) {
   auto plan = std::make_unique<apc::DigestPlan<MAXE>>();
+  plan->one = 1;
   size_t i = 0;
   while (i < entries.size()) {
     const size_t k = std::min(entries.size() - i, (size_t)MAXE);

@@ -76,7 +76,7 @@ struct CommitPlan {
   uint64_t total_tiles;
   uint64_t total_scalar;
   uint32_t count;
-  uint32_t pad_;
+  uint32_t one;          // 1: the FMA-pipe carry-add multiplier of the digest
   CommitEntry e[MAXE];
 };
 
@@ -111,7 +111,7 @@ template <int MAXE>
 struct DigestPlan {
   uint64_t total_tiles;
   uint32_t count;
-  uint32_t pad_;
+  uint32_t one;          // 1: the FMA-pipe carry-add multiplier of the digest
   DigestEntry e[MAXE];
 };
 
