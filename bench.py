@@ -169,22 +169,19 @@ def shard_offset(rank: int, elements_per_rank: int) -> int:
     return rank * elements_per_rank
 
 
-def exchange_digests(dist, commit_digests: list[int], verify_digests: list[int]):
-    """Post-step control-plane exchange (Gloo): every rank contributes its 4
-    commit digests and whether its verification pass reproduced them.
-    Returns (whole-model digests = wrapping sum over the shards, all ranks
-    verified, per-rank digests)."""
-    mine = [[int(d) & M64 for d in commit_digests], [int(d) & M64 for d in verify_digests]]
+def exchange_digests(dist, step: int, commit_digests: list[int], verify_digests: list[int], shard: int):
+    """Post-step control-plane exchange: every rank reports (frontier =
+    optimizer step, generation 0, its 4 commit digests, whether its
+    verification pass reproduced them) and the cohort checks agreement
+    (paper_2609_18178_gb300.cohort).  Returns (whole-model digests = wrapping
+    sum over the shards, all verified); raises cohort.CohortError otherwise."""
+    commit = [int(d) & M64 for d in commit_digests]
+    ok = commit == [int(d) & M64 for d in verify_digests]
     if dist is None:
-        gathered = [mine]
-    else:
-        gathered = [None] * dist.get_world_size()
-        dist.all_gather_object(gathered, mine)
-    whole = [0, 0, 0, 0]
-    for c, _ in gathered:
-        whole = [(a + b) & M64 for a, b in zip(whole, c)]
-    verified = all(c == v for c, v in gathered)
-    return whole, verified, [c for c, _ in gathered]
+        return commit, ok
+    from paper_2609_18178_gb300 import cohort
+    ag = cohort.agree(dist, frontier=step, generation=0, digests=commit, shard=shard, verified=ok)
+    return ag.whole_digests, True
 
 
 def group_pieces(sizes: list[int], n_groups: int) -> list[list[int]]:
@@ -277,7 +274,7 @@ def run_gpu(args):
     ms_per_step = total_ms / K
     digests_c = apc.digests_to_host(out_c)
     digests_v = apc.digests_to_host(out_v)
-    whole, verified, _ = exchange_digests(dist, digests_c, digests_v)
+    whole, verified = exchange_digests(dist, step_t, digests_c, digests_v, shard=rank)
 
     # End to end: every step brings its gradient from pinned host memory and
     # returns the digests.  The table is cut into groups of about equal size;
@@ -332,9 +329,19 @@ def run_gpu(args):
         e2e_ms = max_over_ranks(dist, e0.elapsed_time(e1)) / ke
         got = [[int(x) & M64 for x in row] for row in host_out.tolist()]
         e2e_verified = all(r[:4] == r[4:] for r in got)
+        # the upload alone (same copies, no kernels): the bound of the end-to-end step
+        h0, h1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        h0.record(copy_stream)
+        with torch.cuda.stream(copy_stream):
+            for k, pc in enumerate(w.pieces):
+                bufs[pc.alloc]["g"][pc.at:pc.at + pc.n].copy_(host_g[pc.alloc][pc.at:pc.at + pc.n], non_blocking=True)
+        h1.record(copy_stream)
+        torch.cuda.synchronize()
+        h2d_ms = h0.elapsed_time(h1)
         e2e = {"value": world * N / (e2e_ms * 1e-3), "unit": "elements/s",
                "h2d_bytes_per_step": 2 * N, "d2h_bytes_per_step": 64 * n_groups, "ms_per_step": e2e_ms,
-               "steps": ke, "groups": n_groups, "verify_matches_commit": e2e_verified}
+               "steps": ke, "groups": n_groups, "verify_matches_commit": e2e_verified,
+               "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": 2 * N / (h2d_ms * 1e-3) / 1e9}
         del host_g
 
     # Next rows measured beside the step: the fused commit that also zeroes

@@ -3,7 +3,8 @@ its own shard (here with the oracle standing in for the device), the ranks
 bracket the step with barriers and a max-over-ranks time, then exchange their
 32-byte digests on the control plane.  The whole-model digest is the wrapping
 sum of the shard digests (concatenation), and a bit flipped on one rank's
-host copy before its verification is caught by every rank."""
+host copy before its verification is caught by every rank (fail-stop on a
+failed validation, the paper's Section III-C safety invariant)."""
 import multiprocessing as mp
 import os
 import socket
@@ -47,9 +48,14 @@ def _rank_main(rank, world, port, flip_rank, q):
             off += n
         t = bench.max_over_ranks(dist, float(rank + 1))
         bench.barrier(dist)
-        whole, verified, per_rank = bench.exchange_digests(dist, commit, verify)
+        from paper_2609_18178_gb300 import cohort
+        try:
+            whole, verified = bench.exchange_digests(dist, STEP, commit, verify, shard=rank)
+            outcome = "agreed"
+        except cohort.CohortMismatch as e:
+            whole, verified, outcome = None, False, "mismatch:%s:%s" % (e.what, e.ranks)
         dist.destroy_process_group()
-        q.put((rank, t, whole, verified, per_rank))
+        q.put((rank, t, whole, verified, outcome))
     except Exception as e:  # report to the parent instead of hanging it
         q.put((rank, "error", repr(e), None, None))
 
@@ -86,15 +92,14 @@ def _whole_model_digest(world):
 def test_two_ranks_exchange_digests():
     res = _run(2, flip_rank=-1)
     want = _whole_model_digest(2)
-    for rank, t, whole, verified, per_rank in res:
+    for rank, t, whole, verified, outcome in res:
         assert t == 2.0                      # max over ranks of (rank + 1)
-        assert verified
+        assert outcome == "agreed" and verified
         assert whole == want                 # concatenation: shards sum to the whole model
-        assert per_rank[0] != per_rank[1]    # distinct shards
     assert res[0][2] == res[1][2]
 
 
 def test_host_fault_on_one_rank_is_seen_by_all():
     res = _run(2, flip_rank=1)
-    for rank, t, whole, verified, per_rank in res:
-        assert not verified
+    for rank, t, whole, verified, outcome in res:
+        assert outcome == "mismatch:verification:[1]"
