@@ -47,14 +47,14 @@ def shard_digests(shard, flip=False):
 ROUNDS = [None, "frontier", "flip", "guard"]
 
 
-def _one_round(dist, rank, fault):
+def _one_round(dist, grp, rank, fault):
     shard = rank // 2
     frontier = STEP + (1 if fault == "frontier" and rank == 2 else 0)
     guard = not (fault == "guard" and rank == 1)
     d = shard_digests(shard, flip=(fault == "flip" and rank == 3))
     t0 = time.perf_counter()
     try:
-        ag = cohort.agree(dist, frontier, 1, d, shard, guard_ok=guard)
+        ag = cohort.agree(dist, frontier, 1, d, shard, guard_ok=guard, group=grp)
         return ("agreed", ag.whole_digests, ag.seconds)
     except cohort.CohortMismatch as e:
         return ("mismatch", (e.what, e.ranks), time.perf_counter() - t0)
@@ -66,7 +66,10 @@ def _rank(rank, world, port, rounds, q):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     try:
         import torch.distributed as dist
-        dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=6))
+        # a generous rendezvous (cold imports), then the protocol's own group
+        # whose timeout is its 6 s deadline
+        dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=120))
+        grp = dist.new_group(ranks=list(range(world)), backend="gloo", timeout=datetime.timedelta(seconds=6))
         outcomes = []
         for fault in rounds:
             if fault == "lost" and rank == 3:
@@ -75,7 +78,7 @@ def _rank(rank, world, port, rounds, q):
                 q.join_thread()                              # flush before leaving
                 os._exit(0)                                  # leaves without taking part
             # a mismatch reaches every rank after the exchange, so the group stays usable
-            outcomes.append(_one_round(dist, rank, fault))
+            outcomes.append(_one_round(dist, grp, rank, fault))
         q.put((rank, outcomes))
         try:
             dist.destroy_process_group()
