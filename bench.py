@@ -199,6 +199,108 @@ def group_pieces(sizes: list[int], n_groups: int) -> list[list[int]]:
     return groups
 
 
+# ----------------------------------------------- replica verification (f4)
+
+def _replica_main(idx: int, n_rep: int, port: int, workload: str, flip: int, q) -> None:
+    """One replica of a hybrid-sharding replication group on the current
+    GPU: commit its (identical) shard, then, in two rounds, verify and agree
+    with the other replicas; in round 2 one bit of replica `flip`'s HBM state
+    is flipped first through a host-side copy.  Spawned, so it builds its own
+    CUDA context; replicas never wait on each other's kernels, only on the
+    host control plane."""
+    import datetime
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    try:
+        import torch
+        import torch.distributed as dist
+        import paper_2609_18178_gb300 as apc
+        from paper_2609_18178_gb300 import cohort
+        import synth
+        from synth import workloads as W
+        dist.init_process_group("gloo", rank=idx, world_size=n_rep, timeout=datetime.timedelta(seconds=300))
+        grp = dist.new_group(ranks=list(range(n_rep)), backend="gloo", timeout=datetime.timedelta(seconds=60))
+        torch.cuda.set_device(0)
+        w = W.ALL[workload]()
+        step = w.steps[-1]
+        s = torch.cuda.current_stream().cuda_stream
+        bufs, goff = [], {}
+        for pc in w.pieces:
+            goff.setdefault(pc.alloc, pc.goff - pc.at)
+        for a, n in enumerate(w.allocs):
+            b = {k: torch.empty(n, dtype=torch.float32 if k in "pmv" else torch.int16, device="cuda")
+                 for k in "pmvgw"}
+            for k, kind in (("p", synth.P), ("m", synth.M), ("v", synth.V)):
+                synth.fill_dev(kind, b[k].data_ptr(), n, goff[a], stream=s)
+            synth.fill_dev(synth.G, b["g"].data_ptr(), n, goff[a], step=step, stream=s)
+            bufs.append(b)
+        entries, vbufs = [], []
+        for pc in w.pieces:
+            b = bufs[pc.alloc]
+            sl = slice(pc.at, pc.at + pc.n)
+            entries.append(apc.TensorEntry(b["p"][sl], b["m"][sl], b["v"][sl], b["g"][sl], b["w"][sl], pc.goff))
+            vbufs += apc.state_buffers(b["p"][sl], b["m"][sl], b["v"][sl], b["w"][sl], pc.goff)
+        dc = apc.digests_to_host(apc.commit_step(entries, step, HP))
+        rounds = []
+        for r, flip_here in enumerate((False, idx == flip)):
+            if flip_here:
+                word = bufs[0]["p"][12345:12346].view(torch.int32).cpu()
+                word ^= 1 << 7
+                bufs[0]["p"][12345:12346].view(torch.int32).copy_(word)    # host-side fault injection
+            dist.barrier(group=grp)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            dv = apc.digests_to_host(apc.digest(vbufs, 4))
+            t1 = time.perf_counter()
+            try:
+                ag = cohort.agree(dist, step, 1, dv, shard=0, group=grp)
+                rounds.append(("agreed", ["%016x" % d for d in ag.whole_digests], (t1 - t0) * 1e3,
+                               ag.seconds * 1e3))
+            except cohort.CohortMismatch as e:
+                rounds.append(("mismatch", (e.what, e.ranks), (t1 - t0) * 1e3, (time.perf_counter() - t1) * 1e3))
+        q.put((idx, dc, rounds))
+        dist.destroy_process_group()
+    except Exception as e:  # reported, never hangs the parent
+        q.put((idx, None, "error: %r" % (e,)))
+
+
+def replica_check(n_rep: int = 4, workload: str = "c4", flip: int = 3, timeout_s: float = 600.0) -> dict:
+    """Run the replica verification with n_rep spawned processes on GPU 0."""
+    import multiprocessing as mp
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    ps = [ctx.Process(target=_replica_main, args=(i, n_rep, port, workload, flip, q)) for i in range(n_rep)]
+    t0 = time.perf_counter()
+    for p in ps:
+        p.start()
+    res = []
+    try:
+        for _ in ps:
+            res.append(q.get(timeout=timeout_s))
+    finally:
+        for p in ps:
+            p.join(timeout=60)
+            if p.is_alive():
+                p.kill()
+    res.sort(key=lambda x: x[0])
+    errors = [r[2] for r in res if isinstance(r[2], str)]
+    if errors:
+        return {"replicas": n_rep, "error": errors[0]}
+    commit_equal = all(r[1] == res[0][1] for r in res)
+    ok_round = [r[2][0] for r in res]
+    flip_round = [r[2][1] for r in res]
+    return {"replicas": n_rep, "workload": workload, "commit_digests_equal": commit_equal,
+            "round1_agreed": all(o[0] == "agreed" for o in ok_round),
+            "round2_flip_replica": flip,
+            "round2_detected_by_all": all(o[0] == "mismatch" for o in flip_round),
+            "round2_diagnosis": flip_round[0][1] if flip_round[0][0] == "mismatch" else None,
+            "verify_ms_max": max(o[2] for o in ok_round), "agree_ms_max": max(o[3] for o in ok_round),
+            "wall_s": time.perf_counter() - t0}
+
+
 # ------------------------------------------------------------- GPU arm
 
 def run_gpu(args):
@@ -406,6 +508,14 @@ def run_gpu(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, step_t, args.cpu_seconds)
 
+    if rank == 0 and world == 1 and not args.no_next and args.replicas > 1:
+        # c5 + f3 stay resident (about 160 GB); the replicas add 4 x 7.3 GB
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        f4 = replica_check(args.replicas, "c4", flip=args.replicas - 1)
+        if nxt is not None:
+            nxt["f4_replica_verify"] = f4
+
     if rank != 0:
         if dist is not None:
             dist.destroy_process_group()
@@ -520,7 +630,8 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
-    ap.add_argument("--no-next", action="store_true", help="skip the next-row measurements (zero-grad commit, guard)")
+    ap.add_argument("--no-next", action="store_true", help="skip the next-row measurements (f1, f3, f4)")
+    ap.add_argument("--replicas", type=int, default=4, help="replica processes of the f4 verification (<= 1: skip)")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         print("note: at least 3 warm-up steps are required for a valid number", file=sys.stderr)
