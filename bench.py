@@ -381,8 +381,10 @@ def run_gpu(args):
     # End to end: every step brings its gradient from pinned host memory and
     # returns the digests.  The table is cut into groups of about equal size;
     # a copy stream moves group g's gradient while the compute stream commits
-    # and verifies group g-1 (events order each group's kernels after its
-    # copies), and the host adds the per-group digests (concatenation).
+    # and verifies earlier groups (events order each group's kernels after its
+    # copies, and each upload after the previous step's commit of that group
+    # has read the old gradient), and the host adds the per-group digests
+    # (concatenation).
     e2e = None
     if not args.no_e2e:
         host_g = []
@@ -397,13 +399,13 @@ def run_gpu(args):
         host_out = torch.empty(n_groups, 8, dtype=torch.int64, pin_memory=True)
         ready = [torch.cuda.Event() for _ in range(n_groups)]
         done = [torch.cuda.Event() for _ in range(n_groups)]
-        start_ev = torch.cuda.Event()
         torch.cuda.synchronize()
 
         def e2e_step():
-            start_ev.record(stream)
-            copy_stream.wait_event(start_ev)
+            # group g's upload for this step waits only until the previous
+            # step's commit of group g has read its gradient (done[g])
             for gi, idx in enumerate(groups):
+                copy_stream.wait_event(done[gi])
                 with torch.cuda.stream(copy_stream):
                     for k in idx:
                         pc = w.pieces[k]
@@ -412,6 +414,7 @@ def run_gpu(args):
                     ready[gi].record(copy_stream)
                 stream.wait_event(ready[gi])
                 apc.commit_step([entries[k] for k in idx], step_t, HP, stream=s, out=outs[gi, :4])
+                done[gi].record(stream)
                 apc.digest([vbufs[4 * k + j] for k in idx for j in range(4)], 4, stream=s, out=outs[gi, 4:])
             host_out.copy_(outs, non_blocking=True)
 
@@ -423,6 +426,7 @@ def run_gpu(args):
         barrier(dist)
         torch.cuda.synchronize()
         e0.record(stream)
+        copy_stream.wait_event(e0)
         for _ in range(ke):
             e2e_step()
         e1.record(stream)

@@ -88,9 +88,15 @@ static_assert(sizeof(CommitPlan<kCommitLarge>) <= 32764, "kernel parameter limit
 // Digest kernel: register-staged streaming (the pass is bound by integer
 // issue, so the loads are issued straight from the compute warps: a thread
 // handles kDigestUnroll 8-element vectors per tile).
-constexpr int kThreads = 256;              // threads per CTA of the digest kernel
-constexpr int kDigestUnroll = 4;           // thread-vectors per thread per tile
-constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 8192 elements
+#ifndef APC_DIGEST_THREADS
+#define APC_DIGEST_THREADS 384
+#endif
+#ifndef APC_DIGEST_UNROLL
+#define APC_DIGEST_UNROLL 4
+#endif
+constexpr int kThreads = APC_DIGEST_THREADS;     // threads per CTA of the digest kernel
+constexpr int kDigestUnroll = APC_DIGEST_UNROLL; // thread-vectors per thread per tile
+constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 12,288 elements
 
 // One buffer of the digest kernel (32 bytes).
 //   head: scalar elements before the first 16-byte boundary (<= 7); then
