@@ -527,3 +527,41 @@ def test_f3_rank_shard_bf16_full_size():
     assert part == oracle_workload_digest_bf16(w, 5, lo, hi)
     del dw
     torch.cuda.empty_cache()
+
+
+def test_single_entry_longer_than_2_32_elements():
+    """One entry of 2^32 + 4099 elements (64-bit tile and element indices
+    inside one tensor, ~69 GB of state): sampled elements against the
+    oracle; the same data given as three pieces digests identically; a
+    window around the entry's 2^32nd element matches the streamed oracle."""
+    free, _ = torch.cuda.mem_get_info()
+    if free < 80 * (1 << 30):
+        pytest.skip("needs ~75 GB of free device memory")
+    n = (1 << 32) + 4099
+    goff = 1000
+    w1 = W.Workload("big", [W.Piece("flat", n, goff, 0, 0)], [3], chained=False, allocs=[n])
+    dw = DeviceWorkload(w1, 3)
+    # as three pieces first (ragged cuts), then the state is regenerated and run as one entry
+    cuts = [0, 123_456_789, (1 << 32) - 5, n]
+    b = dw.bufs[0]
+    pieces = [apc.TensorEntry(b["p"][a:c], b["m"][a:c], b["v"][a:c], b["g"][a:c], b["w"][a:c], goff + a)
+              for a, c in zip(cuts[:-1], cuts[1:])]
+    d3 = apc.digests_to_host(apc.commit_step(pieces, 3, HP))
+    dw.fill_state()
+    d1 = apc.digests_to_host(apc.commit_step(dw.entries(), 3, HP))
+    assert d1 == d3
+    idx = np.unique(np.concatenate([sample_indices(w1, 50000, 11),
+                                    np.array([goff + (1 << 32) + j for j in (-2, -1, 0, 1, 4098)], dtype=np.uint64)]))
+    got = dw.gather(idx)
+    ref = oracle_at(idx, 3)
+    for key in "pmvw":
+        assert np.array_equal(got[key], ref[key]), key
+    lo = (1 << 32) - (1 << 20)            # element offsets inside the entry
+    hi = (1 << 32) + 4099
+    sl = slice(lo, hi)
+    part = apc.digests_to_host(apc.digest(apc.state_buffers(b["p"][sl], b["m"][sl], b["v"][sl], b["w"][sl],
+                                                            goff + lo), 4))
+    wpart = W.Workload("win", [W.Piece("win", hi - lo, goff + lo, 0, 0)], [3], chained=False, allocs=[hi - lo])
+    assert part == oracle_workload_digest(wpart, 3)
+    del dw, b, pieces
+    torch.cuda.empty_cache()
