@@ -575,8 +575,11 @@ def run_gpu(args):
 
 def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
     """The oracle (as it stands) on all host cores over a bounded sample: the
-    first ``sample`` elements of the workload's flat order, repeated until
+    first ``sample`` elements of the workload's flat order, one step = the
+    oracle's commit (threaded) then its digests of the four written buffers
+    (the verification pass, chunks on a thread pool), repeated until
     ``seconds`` of work; input generation is not timed."""
+    from concurrent.futures import ThreadPoolExecutor
     import oracle
     import synth
     n = min(sample, w.n)
@@ -585,16 +588,33 @@ def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
     p, m, v = synth.state(n, g0)
     g = synth.grad(n, g0, step_t)
     h8 = oracle.resolve_hparams(HP, step_t)
-    done, t0 = 0, time.perf_counter()
+    chunk = -(-n // cores)
+
+    def verify(wb):
+        parts = []
+        for lo in range(0, n, chunk):
+            hi = min(n, lo + chunk)
+            parts += [(oracle.digest_f32, p[lo:hi], lo), (oracle.digest_f32, m[lo:hi], lo),
+                      (oracle.digest_f32, v[lo:hi], lo), (oracle.digest_u16, wb[lo:hi], lo)]
+        with ThreadPoolExecutor(cores) as ex:
+            res = list(ex.map(lambda a: a[0](a[1], g0 + a[2]), parts))
+        tot = [0, 0, 0, 0]
+        for k, r in enumerate(res):
+            tot[k % 4] = (tot[k % 4] + r) & M64
+        return tot
+
+    done, ok, t0 = 0, True, time.perf_counter()
     while True:
-        oracle.commit(p, m, v, g, g0, h8, nthreads=cores)
+        wb, d = oracle.commit(p, m, v, g, g0, h8, nthreads=cores)
+        ok = ok and verify(wb) == d
         done += n
         el = time.perf_counter() - t0
         if el >= seconds or el * (done + n) / done > 3 * seconds:
             break
     return {"value": done / el, "unit": "elements/s", "cores": cores, "kind": "oracle",
-            "sample": "first %d elements of %s (embed_tokens), step %d, %d passes, %.1f s" % (n, w.name, step_t,
-                                                                                          done // n, el)}
+            "sample": "first %d elements of %s (embed_tokens), step %d (commit + verification digests), "
+                      "%d passes, %.1f s" % (n, w.name, step_t, done // n, el),
+            "verify_matches_commit": ok}
 
 
 def run_reference(args):
