@@ -42,8 +42,9 @@
  *
  * Conventions for every call:
  *   - Device pointers belong to the calling thread's current CUDA device.
- *     The caller owns all memory; the library allocates nothing and keeps
- *     no state between calls.
+ *     The caller owns all memory and the library allocates nothing.  Between
+ *     calls it keeps only each device's SM count and kernel residency
+ *     (queried once) and the kernels' device status word (apc_device_status).
  *   - Work is enqueued on `stream` (NULL = the legacy default stream); the
  *     call never synchronizes.  Results, including the digests, are valid
  *     once the stream reaches that point.
