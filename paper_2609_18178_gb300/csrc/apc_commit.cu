@@ -36,6 +36,8 @@
 // consuming, drains the copies already issued (bounded again) and returns.
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "../../include/apc.h"
 #include "apc_device.cuh"
 #include "apc_internal.h"
@@ -63,6 +65,15 @@ __device__ __forceinline__ uint32_t bf16_rne_bits(float x) {
 
 __device__ __forceinline__ float bf16_value(uint32_t h) { return __uint_as_float(h << 16); }
 
+// A consumer thread's output addresses in the current tile: element
+// start + 4t of the entry (t the consumer index).  Group k of the thread then
+// sits at a compile-time element offset k * 4 * kCommitConsumers, which the
+// stores carry as an immediate.
+struct Dst {
+  void *p, *m, *v;
+  uint16_t *w, *g;
+};
+
 // ------------------------------------------------------------ fp32 state
 
 struct F32State {
@@ -80,10 +91,10 @@ struct F32State {
     r.g = *reinterpret_cast<const uint2 *>(st + 12 * kCommitTile + 2 * e);
   }
 
-  // Four consecutive elements at element i of the entry; G is the digest
-  // index of the first.
-  __device__ static void compute_store(const CommitEntry &E, uint64_t i, uint32_t G, const Regs &r,
-                                       const Scalars &s, Acc &a) {
+  // Four consecutive elements at element offset `off` from the thread's
+  // output addresses; G is the digest index of the first.
+  __device__ static void compute_store(const Dst &d, uint32_t off, uint32_t G, const Regs &r, const Scalars &s,
+                                       Acc &a) {
     float p[4] = {r.p.x, r.p.y, r.p.z, r.p.w};
     float m[4] = {r.m.x, r.m.y, r.m.z, r.m.w};
     float v[4] = {r.v.x, r.v.y, r.v.z, r.v.w};
@@ -91,26 +102,18 @@ struct F32State {
     uint32_t w[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) w[j] = adamw_element(p[j], m[j], v[j], gw[j], s);
-    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.p) + i), make_float4(p[0], p[1], p[2], p[3]));
-    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.m) + i), make_float4(m[0], m[1], m[2], m[3]));
-    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(E.v) + i), make_float4(v[0], v[1], v[2], v[3]));
-    __stcs(reinterpret_cast<uint2 *>(E.w + i), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
-    acc_add(a.p, digest_term(G, __float_as_uint(p[0]), s.one), s.one);
-    acc_add(a.p, digest_term(G + 1, __float_as_uint(p[1]), s.one), s.one);
-    acc_add(a.p, digest_term(G + 2, __float_as_uint(p[2]), s.one), s.one);
-    acc_add(a.p, digest_term(G + 3, __float_as_uint(p[3]), s.one), s.one);
-    acc_add(a.m, digest_term(G, __float_as_uint(m[0]), s.one), s.one);
-    acc_add(a.m, digest_term(G + 1, __float_as_uint(m[1]), s.one), s.one);
-    acc_add(a.m, digest_term(G + 2, __float_as_uint(m[2]), s.one), s.one);
-    acc_add(a.m, digest_term(G + 3, __float_as_uint(m[3]), s.one), s.one);
-    acc_add(a.v, digest_term(G, __float_as_uint(v[0]), s.one), s.one);
-    acc_add(a.v, digest_term(G + 1, __float_as_uint(v[1]), s.one), s.one);
-    acc_add(a.v, digest_term(G + 2, __float_as_uint(v[2]), s.one), s.one);
-    acc_add(a.v, digest_term(G + 3, __float_as_uint(v[3]), s.one), s.one);
-    acc_add(a.w, digest_term(G, w[0], s.one), s.one);
-    acc_add(a.w, digest_term(G + 1, w[1], s.one), s.one);
-    acc_add(a.w, digest_term(G + 2, w[2], s.one), s.one);
-    acc_add(a.w, digest_term(G + 3, w[3], s.one), s.one);
+    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(d.p) + off), make_float4(p[0], p[1], p[2], p[3]));
+    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(d.m) + off), make_float4(m[0], m[1], m[2], m[3]));
+    __stcs(reinterpret_cast<float4 *>(static_cast<float *>(d.v) + off), make_float4(v[0], v[1], v[2], v[3]));
+    __stcs(reinterpret_cast<uint2 *>(d.w + off), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
+    a.p += digest_term(G, __float_as_uint(p[0]), s.one) + digest_term(G + 1, __float_as_uint(p[1]), s.one);
+    a.p += digest_term(G + 2, __float_as_uint(p[2]), s.one) + digest_term(G + 3, __float_as_uint(p[3]), s.one);
+    a.m += digest_term(G, __float_as_uint(m[0]), s.one) + digest_term(G + 1, __float_as_uint(m[1]), s.one);
+    a.m += digest_term(G + 2, __float_as_uint(m[2]), s.one) + digest_term(G + 3, __float_as_uint(m[3]), s.one);
+    a.v += digest_term(G, __float_as_uint(v[0]), s.one) + digest_term(G + 1, __float_as_uint(v[1]), s.one);
+    a.v += digest_term(G + 2, __float_as_uint(v[2]), s.one) + digest_term(G + 3, __float_as_uint(v[3]), s.one);
+    a.w += digest_term(G, w[0], s.one) + digest_term(G + 1, w[1], s.one);
+    a.w += digest_term(G + 2, w[2], s.one) + digest_term(G + 3, w[3], s.one);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -145,8 +148,8 @@ struct BF16State {
     r.g = *reinterpret_cast<const uint2 *>(st + 6 * kCommitTile + 2 * e);
   }
 
-  __device__ static void compute_store(const CommitEntry &E, uint64_t i, uint32_t G, const Regs &r,
-                                       const Scalars &s, Acc &a) {
+  __device__ static void compute_store(const Dst &d, uint32_t off, uint32_t G, const Regs &r, const Scalars &s,
+                                       Acc &a) {
     const uint32_t pw[4] = {r.p.x & 0xFFFFu, r.p.x >> 16, r.p.y & 0xFFFFu, r.p.y >> 16};
     const uint32_t mw[4] = {r.m.x & 0xFFFFu, r.m.x >> 16, r.m.y & 0xFFFFu, r.m.y >> 16};
     const uint32_t vw[4] = {r.v.x & 0xFFFFu, r.v.x >> 16, r.v.y & 0xFFFFu, r.v.y >> 16};
@@ -159,24 +162,18 @@ struct BF16State {
       mo[j] = bf16_rne_bits(m);
       vo[j] = bf16_rne_bits(v);
     }
-    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(E.p) + i),
+    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(d.p) + off),
            make_uint2(po[0] | (po[1] << 16), po[2] | (po[3] << 16)));
-    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(E.m) + i),
+    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(d.m) + off),
            make_uint2(mo[0] | (mo[1] << 16), mo[2] | (mo[3] << 16)));
-    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(E.v) + i),
+    __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(d.v) + off),
            make_uint2(vo[0] | (vo[1] << 16), vo[2] | (vo[3] << 16)));
-    acc_add(a.p, digest_term(G, po[0], s.one), s.one);
-    acc_add(a.p, digest_term(G + 1, po[1], s.one), s.one);
-    acc_add(a.p, digest_term(G + 2, po[2], s.one), s.one);
-    acc_add(a.p, digest_term(G + 3, po[3], s.one), s.one);
-    acc_add(a.m, digest_term(G, mo[0], s.one), s.one);
-    acc_add(a.m, digest_term(G + 1, mo[1], s.one), s.one);
-    acc_add(a.m, digest_term(G + 2, mo[2], s.one), s.one);
-    acc_add(a.m, digest_term(G + 3, mo[3], s.one), s.one);
-    acc_add(a.v, digest_term(G, vo[0], s.one), s.one);
-    acc_add(a.v, digest_term(G + 1, vo[1], s.one), s.one);
-    acc_add(a.v, digest_term(G + 2, vo[2], s.one), s.one);
-    acc_add(a.v, digest_term(G + 3, vo[3], s.one), s.one);
+    a.p += digest_term(G, po[0], s.one) + digest_term(G + 1, po[1], s.one);
+    a.p += digest_term(G + 2, po[2], s.one) + digest_term(G + 3, po[3], s.one);
+    a.m += digest_term(G, mo[0], s.one) + digest_term(G + 1, mo[1], s.one);
+    a.m += digest_term(G + 2, mo[2], s.one) + digest_term(G + 3, mo[3], s.one);
+    a.v += digest_term(G, vo[0], s.one) + digest_term(G + 1, vo[1], s.one);
+    a.v += digest_term(G + 2, vo[2], s.one) + digest_term(G + 3, vo[3], s.one);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -305,13 +302,17 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[stage]);
-      const uint32_t G0 = E.key_base + (uint32_t)start;
+      const uint64_t first = start + 4 * (uint64_t)ct;   // this thread's first element in the tile
+      const Dst d{static_cast<uint8_t *>(E.p) + first * L::kES, static_cast<uint8_t *>(E.m) + first * L::kES,
+                  static_cast<uint8_t *>(E.v) + first * L::kES, L::kDigests == 4 ? E.w + first : nullptr,
+                  const_cast<uint16_t *>(E.g) + first};
+      const uint32_t G1 = E.key_base + (uint32_t)first;
 #pragma unroll
       for (int k = 0; k < kCommitGroups; ++k) {
-        const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
+        const uint32_t off = (uint32_t)(k * kCommitConsumers) * 4;  // compile-time after unrolling
         if (ok[k]) {
-          if (ZERO) __stcs(reinterpret_cast<uint2 *>(const_cast<uint16_t *>(E.g) + start + e), make_uint2(0u, 0u));
-          L::compute_store(E, start + e, G0 + e, r[k], s, a);
+          if (ZERO) __stcs(reinterpret_cast<uint2 *>(d.g + off), make_uint2(0u, 0u));
+          L::compute_store(d, off, G1 + off, r[k], s, a);
         }
       }
       if (++stage == kCommitStages) {
@@ -363,11 +364,28 @@ __global__ void wait_timeout_kernel(uint64_t limit_ns) {
   if (!mbar_wait(&bar, 0, limit_ns)) atomicOr(&g_commit_status, (unsigned)APC_ETIMEOUT);
 }
 
+// The dynamic shared-memory limit of one kernel instantiation, raised once
+// per device (the first launch on a device sets it; later launches, for
+// example inside a stream capture, only enqueue).
+template <class L, int MAXE, bool ZERO>
+int ensure_smem_attribute() {
+  static std::atomic<uint64_t> done_mask{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return (int)e;
+  const uint64_t bit = dev < 64 ? (1ull << dev) : 0;
+  if (bit && (done_mask.load(std::memory_order_acquire) & bit)) return 0;
+  e = cudaFuncSetAttribute(commit_kernel<L, MAXE, ZERO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem_bytes<L>());
+  if (e != cudaSuccess) return (int)e;
+  if (bit) done_mask.fetch_or(bit, std::memory_order_acq_rel);
+  return 0;
+}
+
 template <class L, int MAXE, bool ZERO>
 int launch_t(const CommitPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
-  cudaError_t e = cudaFuncSetAttribute(commit_kernel<L, MAXE, ZERO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem_bytes<L>());
-  if (e != cudaSuccess) return (int)e;
+  int e = ensure_smem_attribute<L, MAXE, ZERO>();
+  if (e) return e;
   commit_kernel<L, MAXE, ZERO><<<grid, kCommitThreads, smem_bytes<L>(), (cudaStream_t)stream>>>(plan, out);
   return (int)cudaGetLastError();
 }
@@ -384,9 +402,8 @@ int launch(const CommitPlan<MAXE> &plan, int layout, bool zero_grad, unsigned gr
 
 template <class L, int MAXE>
 int blocks_per_sm(int *out) {
-  cudaError_t e = cudaFuncSetAttribute(commit_kernel<L, MAXE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem_bytes<L>());
-  if (e != cudaSuccess) return (int)e;
+  int e = ensure_smem_attribute<L, MAXE, false>();
+  if (e) return e;
   return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<L, MAXE, false>, kCommitThreads,
                                                             smem_bytes<L>());
 }

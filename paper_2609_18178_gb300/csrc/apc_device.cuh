@@ -67,7 +67,9 @@ __device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits, ui
   return z ^ (z >> 31);
 }
 
-// acc += z (mod 2^64), with the high half's carry-add on the FMA pipe.
+// acc += z (mod 2^64), with the high half's carry-add on the FMA pipe.  Used
+// for single terms; pairs of terms are summed as acc += a + b, which the
+// compiler folds into one three-input add per 32-bit half.
 __device__ __forceinline__ void acc_add(uint64_t &acc, uint64_t z, uint32_t one) {
   uint32_t alo = (uint32_t)acc, ahi = (uint32_t)(acc >> 32);
   asm("add.cc.u32 %0, %0, %2;\n\t"

@@ -75,14 +75,10 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
       for (int u = 0; u < kDigestUnroll; ++u) {
         if (!ok[u]) continue;
         const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        acc_add(t0, digest_term(G + 0, x[u][0].x, one), one);
-        acc_add(t0, digest_term(G + 1, x[u][0].y, one), one);
-        acc_add(t1, digest_term(G + 2, x[u][0].z, one), one);
-        acc_add(t1, digest_term(G + 3, x[u][0].w, one), one);
-        acc_add(t0, digest_term(G + 4, x[u][1].x, one), one);
-        acc_add(t0, digest_term(G + 5, x[u][1].y, one), one);
-        acc_add(t1, digest_term(G + 6, x[u][1].z, one), one);
-        acc_add(t1, digest_term(G + 7, x[u][1].w, one), one);
+        t0 += digest_term(G + 0, x[u][0].x, one) + digest_term(G + 1, x[u][0].y, one);
+        t1 += digest_term(G + 2, x[u][0].z, one) + digest_term(G + 3, x[u][0].w, one);
+        t0 += digest_term(G + 4, x[u][1].x, one) + digest_term(G + 5, x[u][1].y, one);
+        t1 += digest_term(G + 6, x[u][1].z, one) + digest_term(G + 7, x[u][1].w, one);
       }
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
@@ -98,14 +94,10 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
       for (int u = 0; u < kDigestUnroll; ++u) {
         if (!ok[u]) continue;
         const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        acc_add(t0, digest_term(G + 0, x[u].x & 0xFFFFu, one), one);
-        acc_add(t0, digest_term(G + 1, x[u].x >> 16, one), one);
-        acc_add(t1, digest_term(G + 2, x[u].y & 0xFFFFu, one), one);
-        acc_add(t1, digest_term(G + 3, x[u].y >> 16, one), one);
-        acc_add(t0, digest_term(G + 4, x[u].z & 0xFFFFu, one), one);
-        acc_add(t0, digest_term(G + 5, x[u].z >> 16, one), one);
-        acc_add(t1, digest_term(G + 6, x[u].w & 0xFFFFu, one), one);
-        acc_add(t1, digest_term(G + 7, x[u].w >> 16, one), one);
+        t0 += digest_term(G + 0, x[u].x & 0xFFFFu, one) + digest_term(G + 1, x[u].x >> 16, one);
+        t1 += digest_term(G + 2, x[u].y & 0xFFFFu, one) + digest_term(G + 3, x[u].y >> 16, one);
+        t0 += digest_term(G + 4, x[u].z & 0xFFFFu, one) + digest_term(G + 5, x[u].z >> 16, one);
+        t1 += digest_term(G + 6, x[u].w & 0xFFFFu, one) + digest_term(G + 7, x[u].w >> 16, one);
       }
     }
     if (local == 0) {

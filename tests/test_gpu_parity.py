@@ -565,3 +565,44 @@ def test_single_entry_longer_than_2_32_elements():
     assert part == oracle_workload_digest(wpart, 3)
     del dw, b, pieces
     torch.cuda.empty_cache()
+
+
+def test_step_captured_in_a_cuda_graph_replays_bit_exact():
+    """The step enqueues only a memset and kernel launches on the caller's
+    stream, so it can be captured once and replayed; each replay equals the
+    eager path step for step (chained state) and the oracle."""
+    tensors = [gen(n, off, 4) for n, off in ((70000, 0), (5, 70000), (33333, 70005))]
+    devs, entries = [], []
+    for t in tensors:
+        d = dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=dev(t["g"]),
+                 w=torch.zeros(t["p"].size, dtype=torch.int16, device="cuda"))
+        devs.append(d)
+        entries.append(apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], t["goff"]))
+    vb = [b for e in entries for b in apc.state_buffers(e.p, e.m, e.v, e.w, e.global_offset)]
+    out_c = torch.empty(4, dtype=torch.int64, device="cuda")
+    out_v = torch.empty(4, dtype=torch.int64, device="cuda")
+    apc.commit_step(entries, 4, HP, out=out_c)        # first call: per-device queries happen outside capture
+    torch.cuda.synchronize()
+    for t, d in zip(tensors, devs):                   # back to the generated state
+        for k in "pmv":
+            d[k].copy_(torch.from_numpy(t[k]).cuda())
+    s = torch.cuda.Stream()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(graph, stream=s):
+            apc.commit_step(entries, 4, HP, stream=s, out=out_c)
+            apc.digest(vb, 4, stream=s, out=out_v)
+    torch.cuda.synchronize()
+    for t, d in zip(tensors, devs):                   # capture does not run the work: reset anyway
+        for k in "pmv":
+            d[k].copy_(torch.from_numpy(t[k]).cuda())
+    h8 = oracle.resolve_hparams(HP, 4)
+    ref = [dict(p=t["p"].copy(), m=t["m"].copy(), v=t["v"].copy(), g=t["g"], goff=t["goff"]) for t in tensors]
+    for rep in range(3):                              # three chained steps, all with t = 4
+        graph.replay()
+        torch.cuda.synchronize()
+        ws, dref = oracle.commit_table(ref, h8)
+        for r, wv in zip(ref, ws):
+            r["w"] = wv
+        assert_same(devs, apc.digests_to_host(out_c), ref, dref)
+        assert apc.digests_to_host(out_v) == dref
