@@ -14,9 +14,10 @@ constexpr int kVec = 8;                    // vector granularity: 16 bytes of bf
 constexpr uint32_t kScalarMode = 0xFFFFFFFFu;  // `head` value of an entry run without vectors
 
 // Commit kernel: warp-specialized pipeline.  One producer warp streams each
-// tile of p, m, v (fp32) and g (bf16) into a ring of shared-memory stages with
-// bulk asynchronous copies; kCommitConsumerWarps warps compute from shared
-// memory and store straight to global memory.
+// tile of p, m, v and g into a ring of shared-memory stages with bulk
+// asynchronous copies; kCommitConsumerWarps warps compute from shared memory
+// and store straight to global memory.
+//
 // Pipeline shape (compile-time; the defaults are the measured best on GB300).
 // 19 consumer warps + 1 producer = 20 warps, 5 per SM sub-partition: each
 // sub-partition's 16,384 registers then give 96 per thread with no spills,
@@ -40,10 +41,9 @@ constexpr int kCommitThreads = kCommitConsumers + 32;                   // + the
 constexpr int kCommitGroups = APC_COMMIT_GROUPS;                        // 4-element groups per thread per tile
 constexpr uint64_t kCommitTile = (uint64_t)kCommitConsumers * 4 * kCommitGroups;
 constexpr int kCommitStages = APC_COMMIT_STAGES;
-constexpr uint32_t kCommitStageBytes = (uint32_t)kCommitTile * 14;      // 12 B fp32 state + 2 B grad
-constexpr uint32_t kCommitSmemBytes = kCommitStages * kCommitStageBytes;
 constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
-static_assert(kCommitSmemBytes <= 227 * 1024, "shared memory per CTA");
+// A stage holds one tile of p, m, v and g: 14 bytes per element for fp32
+// state (133 KB per CTA at the defaults), 8 for bf16 state.
 
 // State layouts of the commit kernel.
 constexpr int kLayoutF32 = 0;   // fp32 p, m, v; bf16 g; bf16 copy w
