@@ -54,11 +54,18 @@ def measured_peak():
 
 
 def kernel_source_hash() -> str:
+    """Hash of the kernel sources' code (comments and blank space removed), so
+    that the recorded ncu traffic is dropped whenever the code changes."""
+    import re
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_18178_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(name.encode() + f.read())
+        with open(os.path.join(csrc, name)) as f:
+            code = f.read()
+        code = re.sub(r"/\*.*?\*/", " ", code, flags=re.S)
+        code = re.sub(r"//[^\n]*", " ", code)
+        code = " ".join(code.split())
+        h.update(name.encode() + code.encode())
     return h.hexdigest()[:16]
 
 
@@ -343,15 +350,18 @@ def run_gpu(args):
         vbufs += apc.state_buffers(b["p"][sl], b["m"][sl], b["v"][sl], b["w"][sl], base + pc.goff)
     out_c = torch.empty(4, dtype=torch.int64, device=dev)
     out_v = torch.empty(4, dtype=torch.int64, device=dev)
+    # the table and the buffer list are marshalled once, as a training job
+    # would: no Python work sits between a timed event and its launch
+    tab, vtab = apc.prepare_table(entries), apc.prepare_buffers(vbufs)
     torch.cuda.synchronize()
 
     def one_step(ev=None):
         if ev is not None:
             ev[0].record(stream)
-        apc.commit_step(entries, step_t, HP, stream=s, out=out_c)
+        apc.commit_step(tab, step_t, HP, stream=s, out=out_c)
         if ev is not None:
             ev[1].record(stream)
-        apc.digest(vbufs, 4, stream=s, out=out_v)
+        apc.digest(vtab, 4, stream=s, out=out_v)
         if ev is not None:
             ev[2].record(stream)
 
@@ -399,6 +409,8 @@ def run_gpu(args):
         host_out = torch.empty(n_groups, 8, dtype=torch.int64, pin_memory=True)
         ready = [torch.cuda.Event() for _ in range(n_groups)]
         done = [torch.cuda.Event() for _ in range(n_groups)]
+        gtab = [apc.prepare_table([entries[k] for k in idx]) for idx in groups]
+        gvtab = [apc.prepare_buffers([vbufs[4 * k + j] for k in idx for j in range(4)]) for idx in groups]
         torch.cuda.synchronize()
 
         def e2e_step():
@@ -413,9 +425,9 @@ def run_gpu(args):
                                                                       non_blocking=True)
                     ready[gi].record(copy_stream)
                 stream.wait_event(ready[gi])
-                apc.commit_step([entries[k] for k in idx], step_t, HP, stream=s, out=outs[gi, :4])
+                apc.commit_step(gtab[gi], step_t, HP, stream=s, out=outs[gi, :4])
                 done[gi].record(stream)
-                apc.digest([vbufs[4 * k + j] for k in idx for j in range(4)], 4, stream=s, out=outs[gi, 4:])
+                apc.digest(gvtab[gi], 4, stream=s, out=outs[gi, 4:])
             host_out.copy_(outs, non_blocking=True)
 
         for _ in range(max(1, args.warmup)):
@@ -461,7 +473,8 @@ def run_gpu(args):
     # gradients (2 B/element).  Run last: they leave the gradients zeroed.
     nxt = None
     if not args.no_next:
-        gbufs = [apc.BufferEntry(bufs[pc.alloc]["g"][pc.at:pc.at + pc.n], 0, 0, apc.BF16) for pc in w.pieces]
+        gbufs = apc.prepare_buffers([apc.BufferEntry(bufs[pc.alloc]["g"][pc.at:pc.at + pc.n], 0, 0, apc.BF16)
+                                     for pc in w.pieces])
         out_n = torch.empty(1, dtype=torch.int64, device=dev)
 
         def timed(fn, reps):
@@ -480,7 +493,7 @@ def run_gpu(args):
 
         nz_before = apc.digests_to_host(apc.count_nonzero(gbufs, 1, stream=s, out=out_n))[0]
         guard_ms = timed(lambda: apc.count_nonzero(gbufs, 1, stream=s, out=out_n), max(3, K))
-        zero_ms = timed(lambda: apc.commit_step(entries, step_t, HP, stream=s, out=out_c, zero_grad=True), max(3, K))
+        zero_ms = timed(lambda: apc.commit_step(tab, step_t, HP, stream=s, out=out_c, zero_grad=True), max(3, K))
         nz_after = apc.digests_to_host(apc.count_nonzero(gbufs, 1, stream=s, out=out_n))[0]
         peak_n, _ = measured_peak()
         torch.cuda.synchronize()
@@ -497,12 +510,13 @@ def run_gpu(args):
             sl = slice(pc.at, pc.at + pc.n)
             e3.append(apc.TensorEntryBF16(b3["p"][sl], b3["m"][sl], b3["v"][sl], b3["g"][sl], pc.goff))
             v3 += apc.state_buffers_bf16(b3["p"][sl], b3["m"][sl], b3["v"][sl], pc.goff)
+        e3, v3 = apc.prepare_table(e3), apc.prepare_buffers(v3)
         out3 = torch.empty(3, dtype=torch.int64, device=dev)
         out3v = torch.empty(3, dtype=torch.int64, device=dev)
         f3_ms = timed(lambda: apc.commit_step_bf16(e3, w3.steps[0], HP, stream=s, out=out3), max(3, K))
         f3v_ms = timed(lambda: apc.digest(v3, 3, stream=s, out=out3v), max(3, K))
         f3_ok = apc.digests_to_host(out3) == apc.digests_to_host(out3v)
-        del b3
+        del b3, e3, v3
         nxt = {"f3_commit_bf16_state": {"workload": "rank 1 of 4 of Mistral-7B, %d elements, 77 pieces, bf16 p/m/v"
                                                     % N3, "ms": f3_ms, "gbs": 14 * N3 / (f3_ms * 1e-3) / 1e9,
                                         "frac": 14 * N3 / (f3_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 14,
@@ -519,7 +533,7 @@ def run_gpu(args):
         cpu = cpu_baseline(w, step_t, args.cpu_seconds)
 
     if rank == 0 and world == 1 and not args.no_next and args.replicas > 1:
-        # c5 + f3 stay resident (about 160 GB); the replicas add 4 x 7.3 GB
+        # the c5 state stays resident (116 GB); the replicas add 4 x 7.3 GB
         torch.cuda.synchronize()
         torch.cuda.empty_cache()
         f4 = replica_check(args.replicas, "c4", flip=args.replicas - 1)

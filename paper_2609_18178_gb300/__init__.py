@@ -15,6 +15,9 @@ Entry points mirror the C names:
   read only (post-recovery verification).
 * :func:`resolve_hparams` -> ``apc_resolve_hparams``: the step's binary32
   scalars (host only).
+
+A table or buffer list that is used every step can be marshalled once with
+:func:`prepare_table` / :func:`prepare_buffers` and passed in its place.
 """
 from __future__ import annotations
 
@@ -25,7 +28,8 @@ from typing import Iterable, Sequence
 
 from . import _build
 
-__all__ = ["TensorEntry", "BufferEntry", "ApcError", "commit_step", "digest", "resolve_hparams",
+__all__ = ["TensorEntry", "TensorEntryBF16", "BufferEntry", "PreparedTable", "ApcError", "commit_step",
+           "commit_step_bf16", "digest", "count_nonzero", "prepare_table", "prepare_buffers", "resolve_hparams",
            "library", "lib_path", "F32", "BF16", "DEFAULT_HPARAMS"]
 
 F32, BF16 = 0, 1
@@ -196,62 +200,95 @@ def _out(out, nslots: int, like):
 COMMIT_ZERO_GRAD = 1
 
 
-def commit_step(table: Sequence[TensorEntry], step: int, hparams: dict | None = None, stream=None, out=None,
-                zero_grad: bool = False):
-    """Enqueue the committed AdamW step + digest over ``table`` on ``stream``
-    (``apc_commit_step``, or ``apc_commit_step_ex`` with
-    APC_COMMIT_ZERO_GRAD when ``zero_grad``: the gradients are also zeroed).
+class PreparedTable:
+    """A chunk table or buffer list marshalled once into its C array, for
+    repeated calls over the same buffers (a training job's table does not
+    change between steps).  It keeps references to the tensors it points
+    into, so their memory stays allocated while it lives."""
 
-    Returns the device int64[4] tensor that receives {D_p', D_m', D_v', D_w}
-    (bit patterns of the unsigned digests; see :func:`digests_to_host`)."""
+    def __init__(self, kind: str, arr, count: int, first, keep: list):
+        self.kind, self.arr, self.count, self.first, self._keep = kind, arr, count, first, keep
+
+    def __len__(self) -> int:
+        return self.count
+
+
+def _commit_array(table, kind: str):
+    if isinstance(table, PreparedTable):
+        if table.kind != kind:
+            raise ValueError("prepared table is a %s table, expected %s" % (table.kind, kind))
+        return table.arr, table.count, table.first
     table = list(table)
-    arr = (_Tensor * max(1, len(table)))()
+    if kind == "f32":
+        arr = (_Tensor * max(1, len(table)))()
+        fields = (("p", 4), ("m", 4), ("v", 4), ("g", 2), ("w", 2))
+    else:
+        arr = (_TensorBF16 * max(1, len(table)))()
+        fields = (("p", 2), ("m", 2), ("v", 2), ("g", 2))
     first = None
     for i, t in enumerate(table):
         n = t.count()
-        for name, buf, size in (("p", t.p, 4), ("m", t.m, 4), ("v", t.v, 4), ("g", t.g, 2), ("w", t.w, 2)):
+        ptrs = []
+        for name, size in fields:
+            buf = getattr(t, name)
             if not isinstance(buf, int) and buf is not None and buf.numel() < n:
                 raise ValueError("table[%d].%s has %d < %d elements" % (i, name, buf.numel(), n))
-        arr[i] = _Tensor(_ptr(t.p, 4), _ptr(t.m, 4), _ptr(t.v, 4), _ptr(t.g, 2), _ptr(t.w, 2), n,
-                         int(t.global_offset) & MASK64)
+            ptrs.append(_ptr(buf, size))
+        arr[i] = (_Tensor if kind == "f32" else _TensorBF16)(*ptrs, n, int(t.global_offset) & MASK64)
         if first is None and not isinstance(t.p, int):
             first = t.p
+    return arr, len(table), first
+
+
+def prepare_table(table: Sequence[TensorEntry] | Sequence[TensorEntryBF16]) -> PreparedTable:
+    """Marshal a chunk table once (fp32-state entries for :func:`commit_step`,
+    bf16-state entries for :func:`commit_step_bf16`)."""
+    table = list(table)
+    kind = "bf16" if table and isinstance(table[0], TensorEntryBF16) else "f32"
+    arr, n, first = _commit_array(table, kind)
+    return PreparedTable(kind, arr, n, first, table)
+
+
+def commit_step(table: Sequence[TensorEntry] | PreparedTable, step: int, hparams: dict | None = None, stream=None,
+                out=None, zero_grad: bool = False):
+    """Enqueue the committed AdamW step + digest over ``table`` on ``stream``
+    (``apc_commit_step``, or ``apc_commit_step_ex`` with
+    APC_COMMIT_ZERO_GRAD when ``zero_grad``: the gradients are also zeroed).
+    ``table`` is a list of :class:`TensorEntry` or a :class:`PreparedTable`.
+
+    Returns the device int64[4] tensor that receives {D_p', D_m', D_v', D_w}
+    (bit patterns of the unsigned digests; see :func:`digests_to_host`)."""
+    arr, n, first = _commit_array(table, "f32")
     out = _out(out, 4, first)
     hp = _hp(hparams)
     if zero_grad:
-        _check(library().apc_commit_step_ex(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
+        _check(library().apc_commit_step_ex(ctypes.addressof(arr), n, ctypes.addressof(hp), int(step),
                                             COMMIT_ZERO_GRAD, ctypes.c_void_p(_stream(stream)),
                                             ctypes.c_void_p(_ptr(out, 8))))
     else:
-        _check(library().apc_commit_step(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
+        _check(library().apc_commit_step(ctypes.addressof(arr), n, ctypes.addressof(hp), int(step),
                                          ctypes.c_void_p(_stream(stream)), ctypes.c_void_p(_ptr(out, 8))))
     return out
 
 
-def commit_step_bf16(table: Sequence[TensorEntryBF16], step: int, hparams: dict | None = None, stream=None,
-                     out=None, zero_grad: bool = False):
+def commit_step_bf16(table: Sequence[TensorEntryBF16] | PreparedTable, step: int, hparams: dict | None = None,
+                     stream=None, out=None, zero_grad: bool = False):
     """Enqueue the bf16-state committed step (``apc_commit_step_bf16``).
     Returns the device int64[3] tensor of {D_p', D_m', D_v'}."""
-    table = list(table)
-    arr = (_TensorBF16 * max(1, len(table)))()
-    first = None
-    for i, t in enumerate(table):
-        n = t.count()
-        for name, buf in (("p", t.p), ("m", t.m), ("v", t.v), ("g", t.g)):
-            if not isinstance(buf, int) and buf is not None and buf.numel() < n:
-                raise ValueError("table[%d].%s has %d < %d elements" % (i, name, buf.numel(), n))
-        arr[i] = _TensorBF16(_ptr(t.p, 2), _ptr(t.m, 2), _ptr(t.v, 2), _ptr(t.g, 2), n, int(t.global_offset) & MASK64)
-        if first is None and not isinstance(t.p, int):
-            first = t.p
+    arr, n, first = _commit_array(table, "bf16")
     out = _out(out, 3, first)
     hp = _hp(hparams)
-    _check(library().apc_commit_step_bf16(ctypes.addressof(arr), len(table), ctypes.addressof(hp), int(step),
+    _check(library().apc_commit_step_bf16(ctypes.addressof(arr), n, ctypes.addressof(hp), int(step),
                                           COMMIT_ZERO_GRAD if zero_grad else 0, ctypes.c_void_p(_stream(stream)),
                                           ctypes.c_void_p(_ptr(out, 8))))
     return out
 
 
 def _buffers(buffers):
+    if isinstance(buffers, PreparedTable):
+        if buffers.kind != "buffers":
+            raise ValueError("prepared table is a %s table, expected a buffer list" % buffers.kind)
+        return buffers.arr, buffers.count, buffers.first
     buffers = list(buffers)
     arr = (_Buffer * max(1, len(buffers)))()
     first = None
@@ -269,9 +306,18 @@ def _buffers(buffers):
     return arr, len(buffers), first
 
 
-def digest(buffers: Iterable[BufferEntry], num_slots: int = 4, stream=None, out=None):
-    """Enqueue the read-only digest of ``buffers`` into ``num_slots`` slots
-    (``apc_digest``).  Returns the device int64[num_slots] output tensor."""
+def prepare_buffers(buffers: Iterable[BufferEntry]) -> PreparedTable:
+    """Marshal a buffer list once for :func:`digest` and :func:`count_nonzero`."""
+    buffers = list(buffers)
+    arr, n, first = _buffers(buffers)
+    return PreparedTable("buffers", arr, n, first, buffers)
+
+
+def digest(buffers: Iterable[BufferEntry] | PreparedTable, num_slots: int = 4, stream=None, out=None):
+    """Enqueue the read-only digest of ``buffers`` (a list of
+    :class:`BufferEntry` or a :class:`PreparedTable`) into ``num_slots``
+    slots (``apc_digest``).  Returns the device int64[num_slots] output
+    tensor."""
     arr, n, first = _buffers(buffers)
     out = _out(out, num_slots, first)
     _check(library().apc_digest(ctypes.addressof(arr), n, int(num_slots), ctypes.c_void_p(_stream(stream)),
@@ -279,7 +325,7 @@ def digest(buffers: Iterable[BufferEntry], num_slots: int = 4, stream=None, out=
     return out
 
 
-def count_nonzero(buffers: Iterable[BufferEntry], num_slots: int = 1, stream=None, out=None):
+def count_nonzero(buffers: Iterable[BufferEntry] | PreparedTable, num_slots: int = 1, stream=None, out=None):
     """Enqueue the quiescence guard (``apc_count_nonzero``): per-slot counts
     of nonzero words.  Returns the device int64[num_slots] output tensor."""
     arr, n, first = _buffers(buffers)

@@ -187,3 +187,30 @@ def test_count_nonzero_argument_checks():
     assert cnt([_B(BASE, 16, 0, 3, 0)], 1) == 1
     assert cnt([_B(BASE + 1, 16, 0, 1, 0)], 1) == 2
     assert cnt([_B(BASE, 16, 0, 0, 0)], 1, out=0x10001) == 2
+
+
+def test_prepared_table_marshals_like_the_list():
+    """prepare_table / prepare_buffers build the same C arrays as the list
+    forms, keep their kind, and the library validates them the same way."""
+    e = [apc.TensorEntry(BASE, BASE + (1 << 30), BASE + (2 << 30), BASE + (3 << 30), BASE + (4 << 30), 7, n=100),
+         apc.TensorEntry(BASE + 400, BASE + (1 << 30) + 400, BASE + (2 << 30) + 400, BASE + (3 << 30) + 200,
+                         BASE + (4 << 30) + 200, 107, n=5)]
+    t = apc.prepare_table(e)
+    arr, n, _ = apc._commit_array(e, "f32")
+    assert t.kind == "f32" and len(t) == n == 2 and bytes(t.arr) == bytes(arr)
+    bad = apc.prepare_table([apc.TensorEntry(BASE + 2, BASE + (1 << 30), BASE + (2 << 30), BASE + (3 << 30),
+                                             BASE + (4 << 30), 0, n=8)])
+    with pytest.raises(apc.ApcError) as ei:
+        apc.commit_step(bad, 1, stream=0, out=0x10000)
+    assert ei.value.status == 2
+    with pytest.raises(ValueError):
+        apc.commit_step_bf16(t, 1, stream=0, out=0x10000)
+    with pytest.raises(ValueError):
+        apc.digest(t, 4, stream=0, out=0x10000)
+    b = apc.prepare_buffers([apc.BufferEntry(BASE + 2, 0, 0, apc.F32, n=16)])
+    assert b.kind == "buffers" and len(b) == 1
+    with pytest.raises(apc.ApcError) as ei:
+        apc.digest(b, 4, stream=0, out=0x10000)
+    assert ei.value.status == 2
+    with pytest.raises(ValueError):
+        apc.commit_step(b, 1, stream=0, out=0x10000)

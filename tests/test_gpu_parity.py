@@ -179,6 +179,29 @@ def test_empty_table_and_zero_length_entries():
     assert np.array_equal(host(d["p"], np.uint32), ref[0]["p"].view(np.uint32))
 
 
+def test_prepared_tables_match_the_oracle_over_chained_steps():
+    """A table marshalled once (prepare_table / prepare_buffers) and reused
+    for chained steps gives the oracle's state and digests at every step."""
+    tensors = [gen(n, off, 1) for n, off in ((4999, 0), (8, 4999), (20011, 5007))]
+    entries, devs = [], []
+    for t in tensors:
+        d = dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=dev(t["g"]),
+                 w=torch.zeros(t["p"].size, dtype=torch.int16, device="cuda"))
+        devs.append(d)
+        entries.append(apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], t["goff"]))
+    tab = apc.prepare_table(entries)
+    vtab = apc.prepare_buffers([b for e in entries for b in apc.state_buffers(e.p, e.m, e.v, e.w, e.global_offset)])
+    ref = [dict(p=t["p"].copy(), m=t["m"].copy(), v=t["v"].copy(), g=t["g"], goff=t["goff"]) for t in tensors]
+    for step in (1, 2, 3):
+        got = apc.digests_to_host(apc.commit_step(tab, step, HP))
+        ver = apc.digests_to_host(apc.digest(vtab, 4))
+        ws, dref = oracle.commit_table(ref, oracle.resolve_hparams(HP, step))
+        for r, wv in zip(ref, ws):
+            r["w"] = wv
+        assert got == dref and ver == dref
+        assert_same(devs, got, ref, dref)
+
+
 def test_guard_bands_untouched():
     """Canary words around every buffer stay intact (bounds of the vector
     head, body and tail paths)."""
