@@ -91,10 +91,11 @@ struct F32State {
     r.g = *reinterpret_cast<const uint2 *>(st + 12 * kCommitTile + 2 * e);
   }
 
-  // Four consecutive elements at element offset `off` from the thread's
-  // output addresses; G is the digest index of the first.
-  __device__ static void compute_store(const Dst &d, uint32_t off, uint32_t G, const Regs &r, const Scalars &s,
-                                       Acc &a) {
+  // Four consecutive elements at the compile-time element offset OFF from
+  // the thread's output addresses, whose first element has digest index G.
+  template <uint32_t OFF>
+  __device__ static void compute_store(const Dst &d, uint32_t G, const Regs &r, const Scalars &s, Acc &a) {
+    constexpr uint32_t off = OFF;
     float p[4] = {r.p.x, r.p.y, r.p.z, r.p.w};
     float m[4] = {r.m.x, r.m.y, r.m.z, r.m.w};
     float v[4] = {r.v.x, r.v.y, r.v.z, r.v.w};
@@ -106,14 +107,14 @@ struct F32State {
     __stcs(reinterpret_cast<float4 *>(static_cast<float *>(d.m) + off), make_float4(m[0], m[1], m[2], m[3]));
     __stcs(reinterpret_cast<float4 *>(static_cast<float *>(d.v) + off), make_float4(v[0], v[1], v[2], v[3]));
     __stcs(reinterpret_cast<uint2 *>(d.w + off), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
-    a.p += digest_term(G, __float_as_uint(p[0]), s.one) + digest_term(G + 1, __float_as_uint(p[1]), s.one);
-    a.p += digest_term(G + 2, __float_as_uint(p[2]), s.one) + digest_term(G + 3, __float_as_uint(p[3]), s.one);
-    a.m += digest_term(G, __float_as_uint(m[0]), s.one) + digest_term(G + 1, __float_as_uint(m[1]), s.one);
-    a.m += digest_term(G + 2, __float_as_uint(m[2]), s.one) + digest_term(G + 3, __float_as_uint(m[3]), s.one);
-    a.v += digest_term(G, __float_as_uint(v[0]), s.one) + digest_term(G + 1, __float_as_uint(v[1]), s.one);
-    a.v += digest_term(G + 2, __float_as_uint(v[2]), s.one) + digest_term(G + 3, __float_as_uint(v[3]), s.one);
-    a.w += digest_term(G, w[0], s.one) + digest_term(G + 1, w[1], s.one);
-    a.w += digest_term(G + 2, w[2], s.one) + digest_term(G + 3, w[3], s.one);
+    a.p += digest_term<OFF>(G, __float_as_uint(p[0]), s.one) + digest_term<OFF + 1>(G, __float_as_uint(p[1]), s.one);
+    a.p += digest_term<OFF + 2>(G, __float_as_uint(p[2]), s.one) + digest_term<OFF + 3>(G, __float_as_uint(p[3]), s.one);
+    a.m += digest_term<OFF>(G, __float_as_uint(m[0]), s.one) + digest_term<OFF + 1>(G, __float_as_uint(m[1]), s.one);
+    a.m += digest_term<OFF + 2>(G, __float_as_uint(m[2]), s.one) + digest_term<OFF + 3>(G, __float_as_uint(m[3]), s.one);
+    a.v += digest_term<OFF>(G, __float_as_uint(v[0]), s.one) + digest_term<OFF + 1>(G, __float_as_uint(v[1]), s.one);
+    a.v += digest_term<OFF + 2>(G, __float_as_uint(v[2]), s.one) + digest_term<OFF + 3>(G, __float_as_uint(v[3]), s.one);
+    a.w += digest_term<OFF>(G, w[0], s.one) + digest_term<OFF + 1>(G, w[1], s.one);
+    a.w += digest_term<OFF + 2>(G, w[2], s.one) + digest_term<OFF + 3>(G, w[3], s.one);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -148,8 +149,9 @@ struct BF16State {
     r.g = *reinterpret_cast<const uint2 *>(st + 6 * kCommitTile + 2 * e);
   }
 
-  __device__ static void compute_store(const Dst &d, uint32_t off, uint32_t G, const Regs &r, const Scalars &s,
-                                       Acc &a) {
+  template <uint32_t OFF>
+  __device__ static void compute_store(const Dst &d, uint32_t G, const Regs &r, const Scalars &s, Acc &a) {
+    constexpr uint32_t off = OFF;
     const uint32_t pw[4] = {r.p.x & 0xFFFFu, r.p.x >> 16, r.p.y & 0xFFFFu, r.p.y >> 16};
     const uint32_t mw[4] = {r.m.x & 0xFFFFu, r.m.x >> 16, r.m.y & 0xFFFFu, r.m.y >> 16};
     const uint32_t vw[4] = {r.v.x & 0xFFFFu, r.v.x >> 16, r.v.y & 0xFFFFu, r.v.y >> 16};
@@ -168,12 +170,12 @@ struct BF16State {
            make_uint2(mo[0] | (mo[1] << 16), mo[2] | (mo[3] << 16)));
     __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(d.v) + off),
            make_uint2(vo[0] | (vo[1] << 16), vo[2] | (vo[3] << 16)));
-    a.p += digest_term(G, po[0], s.one) + digest_term(G + 1, po[1], s.one);
-    a.p += digest_term(G + 2, po[2], s.one) + digest_term(G + 3, po[3], s.one);
-    a.m += digest_term(G, mo[0], s.one) + digest_term(G + 1, mo[1], s.one);
-    a.m += digest_term(G + 2, mo[2], s.one) + digest_term(G + 3, mo[3], s.one);
-    a.v += digest_term(G, vo[0], s.one) + digest_term(G + 1, vo[1], s.one);
-    a.v += digest_term(G + 2, vo[2], s.one) + digest_term(G + 3, vo[3], s.one);
+    a.p += digest_term<OFF>(G, po[0], s.one) + digest_term<OFF + 1>(G, po[1], s.one);
+    a.p += digest_term<OFF + 2>(G, po[2], s.one) + digest_term<OFF + 3>(G, po[3], s.one);
+    a.m += digest_term<OFF>(G, mo[0], s.one) + digest_term<OFF + 1>(G, mo[1], s.one);
+    a.m += digest_term<OFF + 2>(G, mo[2], s.one) + digest_term<OFF + 3>(G, mo[3], s.one);
+    a.v += digest_term<OFF>(G, vo[0], s.one) + digest_term<OFF + 1>(G, vo[1], s.one);
+    a.v += digest_term<OFF + 2>(G, vo[2], s.one) + digest_term<OFF + 3>(G, vo[3], s.one);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -190,6 +192,21 @@ struct BF16State {
     acc_add(a.v, digest_term(G, vo, s.one), s.one);
   }
 };
+
+// Group K of a consumer thread's tile: its elements sit at the compile-time
+// offset K * 4 * kCommitConsumers from the thread's output addresses, which
+// the stores carry as immediates and the digest terms fold into their
+// increment.
+template <class L, bool ZERO, int K>
+__device__ __forceinline__ void store_groups(const Dst &d, uint32_t G1, const typename L::Regs *r, const bool *ok,
+                                             const Scalars &s, Acc &a) {
+  constexpr uint32_t off = (uint32_t)(K * kCommitConsumers) * 4;
+  if (ok[K]) {
+    if (ZERO) __stcs(reinterpret_cast<uint2 *>(d.g + off), make_uint2(0u, 0u));
+    L::template compute_store<off>(d, G1, r[K], s, a);
+  }
+  if constexpr (K + 1 < kCommitGroups) store_groups<L, ZERO, K + 1>(d, G1, r, ok, s, a);
+}
 
 template <class L>
 __host__ __device__ constexpr uint32_t stage_bytes() {
@@ -307,14 +324,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
                   static_cast<uint8_t *>(E.v) + first * L::kES, L::kDigests == 4 ? E.w + first : nullptr,
                   const_cast<uint16_t *>(E.g) + first};
       const uint32_t G1 = E.key_base + (uint32_t)first;
-#pragma unroll
-      for (int k = 0; k < kCommitGroups; ++k) {
-        const uint32_t off = (uint32_t)(k * kCommitConsumers) * 4;  // compile-time after unrolling
-        if (ok[k]) {
-          if (ZERO) __stcs(reinterpret_cast<uint2 *>(d.g + off), make_uint2(0u, 0u));
-          L::compute_store(d, off, G1 + off, r[k], s, a);
-        }
-      }
+      store_groups<L, ZERO, 0>(d, G1, r, ok, s, a);
       if (++stage == kCommitStages) {
         stage = 0;
         phase ^= 1;

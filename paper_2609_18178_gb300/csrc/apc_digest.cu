@@ -23,6 +23,13 @@
 namespace apc {
 namespace {
 
+// One digest term of this pass.  The pass is bound by the integer ALU, not
+// by issue, and runs faster with the compiler's own 64-bit multiply.
+template <uint32_t K>
+__device__ __forceinline__ uint64_t term(uint32_t gidx, uint32_t bits, uint32_t one) {
+  return digest_term<K, MulCompiler>(gidx, bits, one);
+}
+
 __device__ __forceinline__ void flush(uint64_t &acc, int slot, unsigned long long *s_acc) {
   uint64_t x = acc;
 #pragma unroll
@@ -75,10 +82,10 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
       for (int u = 0; u < kDigestUnroll; ++u) {
         if (!ok[u]) continue;
         const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        t0 += digest_term(G + 0, x[u][0].x, one) + digest_term(G + 1, x[u][0].y, one);
-        t1 += digest_term(G + 2, x[u][0].z, one) + digest_term(G + 3, x[u][0].w, one);
-        t0 += digest_term(G + 4, x[u][1].x, one) + digest_term(G + 5, x[u][1].y, one);
-        t1 += digest_term(G + 6, x[u][1].z, one) + digest_term(G + 7, x[u][1].w, one);
+        t0 += term<0>(G, x[u][0].x, one) + term<1>(G, x[u][0].y, one);
+        t1 += term<2>(G, x[u][0].z, one) + term<3>(G, x[u][0].w, one);
+        t0 += term<4>(G, x[u][1].x, one) + term<5>(G, x[u][1].y, one);
+        t1 += term<6>(G, x[u][1].z, one) + term<7>(G, x[u][1].w, one);
       }
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
@@ -94,18 +101,18 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
       for (int u = 0; u < kDigestUnroll; ++u) {
         if (!ok[u]) continue;
         const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        t0 += digest_term(G + 0, x[u].x & 0xFFFFu, one) + digest_term(G + 1, x[u].x >> 16, one);
-        t1 += digest_term(G + 2, x[u].y & 0xFFFFu, one) + digest_term(G + 3, x[u].y >> 16, one);
-        t0 += digest_term(G + 4, x[u].z & 0xFFFFu, one) + digest_term(G + 5, x[u].z >> 16, one);
-        t1 += digest_term(G + 6, x[u].w & 0xFFFFu, one) + digest_term(G + 7, x[u].w >> 16, one);
+        t0 += term<0>(G, x[u].x & 0xFFFFu, one) + term<1>(G, x[u].x >> 16, one);
+        t1 += term<2>(G, x[u].y & 0xFFFFu, one) + term<3>(G, x[u].y >> 16, one);
+        t0 += term<4>(G, x[u].z & 0xFFFFu, one) + term<5>(G, x[u].z >> 16, one);
+        t1 += term<6>(G, x[u].w & 0xFFFFu, one) + term<7>(G, x[u].w >> 16, one);
       }
     }
     if (local == 0) {
       const uint32_t t = threadIdx.x;
-      if (t < head) { acc_add(t0, digest_term(E.key_base + t, word_at(E, t), one), one); }
+      if (t < head) { acc_add(t0, term<0>(E.key_base + t, word_at(E, t), one), one); }
       if (t >= 32 && t - 32 < E.n - vec_end) {
         const uint64_t i = vec_end + (t - 32);
-        acc_add(t0, digest_term(E.key_base + (uint32_t)i, word_at(E, i), one), one);
+        acc_add(t0, term<0>(E.key_base + (uint32_t)i, word_at(E, i), one), one);
       }
     }
     acc_add(acc, t0, one);
