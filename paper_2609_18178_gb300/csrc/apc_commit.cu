@@ -17,8 +17,12 @@
 //    stage is free and issues four bulk asynchronous copies -- p, m, v and g
 //    -- that complete on the stage's "full" mbarrier.  Loads never occupy
 //    consumer registers, and up to kCommitStages tiles per CTA are in flight.
-//  * The consumer warps (19 by default) wait for a stage, read their
-//    elements from shared memory (thread t of C takes elements 4t..4t+3 and
+//  * With each stage the producer also writes a 48-byte descriptor (the
+//    tile's first-element addresses in p, m, v, w, g, its element count and
+//    first digest index) into shared memory before arming the stage, so the
+//    consumers never search the chunk table themselves.
+//  * The consumer warps (19 by default) wait for a stage, read its
+//    descriptor and their elements from shared memory (thread t of C takes elements 4t..4t+3 and
 //    4C+4t..4C+4t+3, so both the shared-memory reads and the global stores
 //    are contiguous across the warp), release the stage to the producer, then
 //    apply AdamW, store the results with streaming stores, and fold the
@@ -73,6 +77,18 @@ struct Dst {
   void *p, *m, *v;
   uint16_t *w, *g;
 };
+
+// What the consumers need of a stage's tile, written into shared memory by
+// the producer before it arms the stage's "full" barrier (whose completion
+// makes it visible to them): the addresses of the tile's first element in
+// p, m, v, w and g, its element count and its first digest index.  The
+// consumers then spend no instructions locating the tile in the chunk table.
+struct __align__(16) StageDesc {
+  uint8_t *p, *m, *v;
+  uint16_t *w, *g;
+  uint32_t cnt, G;
+};
+static_assert(sizeof(StageDesc) == 48, "three 16-byte shared-memory loads");
 
 // ------------------------------------------------------------ fp32 state
 
@@ -232,6 +248,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ __align__(8) uint64_t full[kCommitStages];
   __shared__ __align__(8) uint64_t empty[kCommitStages];
+  __shared__ StageDesc desc[kCommitStages];
   __shared__ uint64_t red[kCommitThreads / 32];
   __shared__ int abort_flag;
 
@@ -266,6 +283,13 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
           break;
         }
         uint8_t *st = smem + (size_t)stage * stage_bytes<L>();
+        desc[stage] = StageDesc{static_cast<uint8_t *>(E.p) + start * L::kES,
+                                static_cast<uint8_t *>(E.m) + start * L::kES,
+                                static_cast<uint8_t *>(E.v) + start * L::kES,
+                                L::kDigests == 4 ? E.w + start : nullptr,
+                                const_cast<uint16_t *>(E.g) + start,
+                                cnt,
+                                E.key_base + (uint32_t)start};
         mbar_arrive_expect_tx(&full[stage], cnt * (3 * L::kES + 2));
         bulk_g2s(st, static_cast<const uint8_t *>(E.p) + start * L::kES, cnt * L::kES, &full[stage], policy);
         bulk_g2s(st + L::kES * kCommitTile, static_cast<const uint8_t *>(E.m) + start * L::kES, cnt * L::kES,
@@ -295,36 +319,31 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
     // ----------------------------------------------------------- consumers
     const Scalars s{plan.h, plan.one};
     const int ct = threadIdx.x;  // 0 .. kCommitConsumers-1
-    uint32_t cur = 0, phase = 0;
+    uint32_t phase = 0;
     int stage = 0;
     for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
-      cur = find_tile(plan, cur, tile);
-      const CommitEntry &E = plan.e[cur];
-      const uint64_t start = E.head + (tile - E.tile_begin) * kCommitTile;
-      const uint64_t vec_end = E.head + ((E.n - E.head) & ~(uint64_t)7);
-      const uint32_t cnt = (uint32_t)umin64(kCommitTile, vec_end - start);
       if (!mbar_wait(&full[stage], phase)) {
         fail_wait(&abort_flag);
         break;
       }
       if (*(volatile int *)&abort_flag) break;
+      const StageDesc sd = desc[stage];
       const uint8_t *st = smem + (size_t)stage * stage_bytes<L>();
       typename L::Regs r[kCommitGroups];
       bool ok[kCommitGroups];
 #pragma unroll
       for (int k = 0; k < kCommitGroups; ++k) {
         const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
-        ok[k] = e < cnt;
+        ok[k] = e < sd.cnt;
         if (ok[k]) L::load(st, e, r[k]);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[stage]);
-      const uint64_t first = start + 4 * (uint64_t)ct;   // this thread's first element in the tile
-      const Dst d{static_cast<uint8_t *>(E.p) + first * L::kES, static_cast<uint8_t *>(E.m) + first * L::kES,
-                  static_cast<uint8_t *>(E.v) + first * L::kES, L::kDigests == 4 ? E.w + first : nullptr,
-                  const_cast<uint16_t *>(E.g) + first};
-      const uint32_t G1 = E.key_base + (uint32_t)first;
-      store_groups<L, ZERO, 0>(d, G1, r, ok, s, a);
+      // this thread's first element in the tile is element 4 * ct
+      const uint32_t ob = 4u * (uint32_t)ct;
+      const Dst d{sd.p + ob * L::kES, sd.m + ob * L::kES, sd.v + ob * L::kES,
+                  L::kDigests == 4 ? sd.w + ob : nullptr, sd.g + ob};
+      store_groups<L, ZERO, 0>(d, sd.G + ob, r, ok, s, a);
       if (++stage == kCommitStages) {
         stage = 0;
         phase ^= 1;
@@ -332,7 +351,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
     }
     // scalar items: entry heads and tails, and entries without vectors
     if (!*(volatile int *)&abort_flag) {
-      cur = 0;
+      uint32_t cur = 0;
       for (uint64_t it = (uint64_t)blockIdx.x * kCommitConsumers + ct; it < plan.total_scalar;
            it += (uint64_t)gridDim.x * kCommitConsumers) {
         while (cur + 1 < plan.count && it >= plan.e[cur + 1].scalar_begin) ++cur;
