@@ -53,6 +53,11 @@
  *   - Errors are returned, never raised: no call aborts the process.  On an
  *     error before launch nothing is enqueued.  apc_last_error() gives a
  *     human-readable detail of the calling thread's last failure.
+ *   - Every kernel runs a persistent grid of (SM count x residency) CTAs, or
+ *     fewer when there is less work.  The environment variable
+ *     APC_GRID_LIMIT, if set to a positive integer when a call is made, caps
+ *     that grid (for tests of grid independence and for sharing the GPU);
+ *     results do not depend on it.
  */
 #ifndef APC_H
 #define APC_H

@@ -12,6 +12,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <memory>
 #include <mutex>
@@ -124,8 +125,15 @@ apc_status device_info(Device *out) {
   return APC_OK;
 }
 
+// The persistent grid: one CTA per resident slot, capped by APC_GRID_LIMIT
+// (read at every call) when that is a positive integer.
 unsigned grid_for(uint64_t tiles, int sms, int per_sm) {
   uint64_t cap = (uint64_t)sms * (uint64_t)std::max(per_sm, 1);
+  if (const char *lim = std::getenv("APC_GRID_LIMIT")) {
+    char *end = nullptr;
+    const unsigned long long v = std::strtoull(lim, &end, 10);
+    if (end != lim && *end == 0 && v > 0) cap = std::min<uint64_t>(cap, v);
+  }
   return (unsigned)std::max<uint64_t>(1, std::min(tiles, cap));
 }
 

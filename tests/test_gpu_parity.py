@@ -367,6 +367,53 @@ def test_repeat_runs_identical():
     torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("limit", [None, 1, 7, 64])
+def test_grid_size_does_not_change_results(monkeypatch, limit):
+    """The same step on persistent grids of 1, 7, 64 CTAs and the default
+    (APC_GRID_LIMIT caps the grid): outputs and digests equal the oracle's,
+    and so does the verification digest on the same grid."""
+    if limit is None:
+        monkeypatch.delenv("APC_GRID_LIMIT", raising=False)
+    else:
+        monkeypatch.setenv("APC_GRID_LIMIT", str(limit))
+    tensors = [gen(n, off, 4) for n, off in ((600_001, (1 << 32) - 300_000), (5, 900_000), (448_570, 1_000_000))]
+    devs, dgot, ref, dref = run_small(tensors, 4)
+    assert_same(devs, dgot, ref, dref)
+    bufs = [b for d, t in zip(devs, tensors) for b in apc.state_buffers(d["p"], d["m"], d["v"], d["w"], t["goff"])]
+    assert apc.digests_to_host(apc.digest(bufs, 4)) == dref
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_single_bit_flip_changes_digest_by_its_term(dtype):
+    """A bit flipped in device memory (through a host copy) changes the
+    digest by exactly splitmix64(new key) - splitmix64(old key) mod 2^64,
+    for every bit position of the word."""
+    rng = np.random.default_rng(21)
+    n, goff = 10_007, (1 << 32) - 5_000
+    if dtype == "f32":
+        udt, sdt, bits, kind = np.uint32, np.int32, 32, apc.F32
+    else:
+        udt, sdt, bits, kind = np.uint16, np.int16, 16, apc.BF16
+    a = rng.integers(0, 1 << bits, size=n, dtype=np.uint64).astype(udt)
+    t = torch.from_numpy(a.view(sdt)).cuda()
+    buf = [apc.BufferEntry(t, 0, goff, kind)]
+    base = apc.digests_to_host(apc.digest(buf, 1))[0]
+    assert base == (oracle.digest_f32(a, goff) if dtype == "f32" else oracle.digest_u16(a, goff))
+    for b in range(bits):
+        i = int(rng.integers(0, n))
+        old = int(a[i])
+        new = old ^ (1 << b)
+        flipped = a.copy()
+        flipped[i] = new
+        t.copy_(torch.from_numpy(flipped.view(sdt)))          # the flip reaches HBM through a host copy
+        got = apc.digests_to_host(apc.digest(buf, 1))[0]
+        key = ((goff + i) & 0xFFFFFFFF) << 32
+        delta = (oracle.splitmix64(key | new) - oracle.splitmix64(key | old)) & M64
+        assert delta != 0 and got == (base + delta) & M64, (b, i)
+    t.copy_(torch.from_numpy(a.view(sdt)))
+    assert apc.digests_to_host(apc.digest(buf, 1))[0] == base
+
+
 def test_bounded_wait_gives_up_and_context_stays_usable():
     """A kernel wait that nothing completes expires (about 50 ms and 2^20
     polls), records APC_ETIMEOUT, and the next committed step still runs
