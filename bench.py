@@ -392,9 +392,12 @@ def run_gpu(args):
     # returns the digests.  The table is cut into groups of about equal size;
     # a copy stream moves group g's gradient while the compute stream commits
     # and verifies earlier groups (events order each group's kernels after its
-    # copies, and each upload after the previous step's commit of that group
+    # upload, and each upload after the previous step's commit of that group
     # has read the old gradient), and the host adds the per-group digests
-    # (concatenation).
+    # (concatenation).  By default the upload is apc_upload: a few CTAs load
+    # the pinned host gradient over the host link, on SMs that the step's
+    # kernels leave free (apc_set_reserved_sms); --e2e-upload copy uses the
+    # DMA copy engines (cudaMemcpyAsync per tensor) instead.
     e2e = None
     if not args.no_e2e:
         host_g = []
@@ -411,29 +414,45 @@ def run_gpu(args):
         done = [torch.cuda.Event() for _ in range(n_groups)]
         gtab = [apc.prepare_table([entries[k] for k in idx]) for idx in groups]
         gvtab = [apc.prepare_buffers([vbufs[4 * k + j] for k in idx for j in range(4)]) for idx in groups]
-        torch.cuda.synchronize()
+
+        def segments(idx):
+            return [apc.Segment(bufs[w.pieces[k].alloc]["g"][w.pieces[k].at:w.pieces[k].at + w.pieces[k].n],
+                                host_g[w.pieces[k].alloc][w.pieces[k].at:w.pieces[k].at + w.pieces[k].n])
+                    for k in idx]
+
+        gseg = [apc.prepare_segments(segments(idx)) for idx in groups]
+        use_sm = args.e2e_upload == "sm"
+
+        def upload(gi, idx):
+            if use_sm:
+                apc.upload(gseg[gi], args.e2e_upload_ctas, stream=copy_stream)
+                return
+            with torch.cuda.stream(copy_stream):
+                for k in idx:
+                    pc = w.pieces[k]
+                    bufs[pc.alloc]["g"][pc.at:pc.at + pc.n].copy_(host_g[pc.alloc][pc.at:pc.at + pc.n],
+                                                                  non_blocking=True)
 
         def e2e_step():
             # group g's upload for this step waits only until the previous
             # step's commit of group g has read its gradient (done[g])
             for gi, idx in enumerate(groups):
                 copy_stream.wait_event(done[gi])
-                with torch.cuda.stream(copy_stream):
-                    for k in idx:
-                        pc = w.pieces[k]
-                        bufs[pc.alloc]["g"][pc.at:pc.at + pc.n].copy_(host_g[pc.alloc][pc.at:pc.at + pc.n],
-                                                                      non_blocking=True)
-                    ready[gi].record(copy_stream)
+                upload(gi, idx)
+                ready[gi].record(copy_stream)
                 stream.wait_event(ready[gi])
                 apc.commit_step(gtab[gi], step_t, HP, stream=s, out=outs[gi, :4])
                 done[gi].record(stream)
                 apc.digest(gvtab[gi], 4, stream=s, out=outs[gi, 4:])
             host_out.copy_(outs, non_blocking=True)
 
+        if use_sm:
+            apc.set_reserved_sms(args.e2e_reserved_sms)
+        torch.cuda.synchronize()
         for _ in range(max(1, args.warmup)):
             e2e_step()
         torch.cuda.synchronize()
-        ke = max(1, min(K, args.e2e_steps))
+        ke = max(1, args.e2e_steps)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         barrier(dist)
         torch.cuda.synchronize()
@@ -446,26 +465,41 @@ def run_gpu(args):
         e1.record(stream)
         torch.cuda.synchronize()
         barrier(dist)
+        apc.set_reserved_sms(0)
         e2e_ms = max_over_ranks(dist, e0.elapsed_time(e1)) / ke
         step_ms = [e0.elapsed_time(step_ev[0])] + [step_ev[k - 1].elapsed_time(step_ev[k]) for k in range(1, ke)]
         got = [[int(x) & M64 for x in row] for row in host_out.tolist()]
         e2e_verified = all(r[:4] == r[4:] for r in got)
-        # the upload alone (same copies, no kernels): the bound of the end-to-end step
-        h0, h1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        h0.record(copy_stream)
-        with torch.cuda.stream(copy_stream):
-            for k, pc in enumerate(w.pieces):
-                bufs[pc.alloc]["g"][pc.at:pc.at + pc.n].copy_(host_g[pc.alloc][pc.at:pc.at + pc.n], non_blocking=True)
-        h1.record(copy_stream)
-        torch.cuda.synchronize()
-        h2d_ms = h0.elapsed_time(h1)
+
+        def upload_alone(sm):
+            # the whole gradient with nothing else running: the bound of the end-to-end step
+            h0, h1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            h0.record(copy_stream)
+            if sm:
+                apc.upload(apc.prepare_segments(segments(range(len(w.pieces)))), args.e2e_upload_ctas,
+                           stream=copy_stream)
+            else:
+                with torch.cuda.stream(copy_stream):
+                    for pc in w.pieces:
+                        bufs[pc.alloc]["g"][pc.at:pc.at + pc.n].copy_(host_g[pc.alloc][pc.at:pc.at + pc.n],
+                                                                      non_blocking=True)
+            h1.record(copy_stream)
+            torch.cuda.synchronize()
+            return h0.elapsed_time(h1)
+
+        h2d_ms = upload_alone(use_sm)
+        ce_ms = upload_alone(False) if use_sm else h2d_ms
         e2e = {"value": world * N / (e2e_ms * 1e-3), "unit": "elements/s",
                "h2d_bytes_per_step": 2 * N, "d2h_bytes_per_step": 64 * n_groups, "ms_per_step": e2e_ms,
                "steps": ke, "groups": n_groups, "verify_matches_commit": e2e_verified,
+               "upload": ({"method": "apc_upload: SM loads of pinned host memory over the host link",
+                           "ctas": args.e2e_upload_ctas, "reserved_sms": args.e2e_reserved_sms} if use_sm else
+                          {"method": "cudaMemcpyAsync per tensor (DMA copy engines)"}),
                "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": 2 * N / (h2d_ms * 1e-3) / 1e9,
+               "copy_engine_alone_ms": ce_ms,
                "step_ms": [round(x, 2) for x in step_ms], "median_step_ms": statistics.median(step_ms),
-               "note": "the host link is shared with other tenants of the machine; steady-state steps sit at "
-                       "the upload-alone time, and bursts of outside traffic lengthen some steps"}
+               "note": "copy-engine transfers on this machine stall for tens to hundreds of ms about twice a "
+                       "second; SM loads over the host link do not"}
         del host_g
 
     # Next rows measured beside the step: the fused commit that also zeroes
@@ -670,6 +704,10 @@ def main(argv=None):
     ap.add_argument("--workload", choices=["c1", "c2", "c3", "c4", "c5"], default="c5")
     ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--e2e-groups", type=int, default=12)
+    ap.add_argument("--e2e-upload", choices=["sm", "copy"], default="sm",
+                    help="end-to-end upload: apc_upload on a few CTAs, or the DMA copy engines")
+    ap.add_argument("--e2e-upload-ctas", type=int, default=16)
+    ap.add_argument("--e2e-reserved-sms", type=int, default=8)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -44,7 +44,8 @@
  *   - Device pointers belong to the calling thread's current CUDA device.
  *     The caller owns all memory and the library allocates nothing.  Between
  *     calls it keeps only each device's SM count and kernel residency
- *     (queried once) and the kernels' device status word (apc_device_status).
+ *     (queried once), the kernels' device status word (apc_device_status)
+ *     and the number of SMs to leave free (apc_set_reserved_sms).
  *   - Work is enqueued on `stream` (NULL = the legacy default stream); the
  *     call never synchronizes.  Results, including the digests, are valid
  *     once the stream reaches that point.
@@ -196,6 +197,42 @@ apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs, int32_t n
  * 1/sqrt(1-b2^t).  Host only; no CUDA call.  out: host, 8 floats. */
 apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t step, float out[8]);
 
+/* One segment of apc_upload: `bytes` bytes from `src` to `dst`.
+ *   dst  device (or managed) memory of the current device, written
+ *   src  memory the device can read: page-locked host memory mapped for the
+ *        device (cudaHostAlloc, cudaHostRegister), pageable host memory on
+ *        devices that read it through the host's page tables
+ *        (cudaDevAttrPageableMemoryAccess), or device memory */
+typedef struct apc_segment {
+  void *dst;
+  const void *src;
+  uint64_t bytes;
+} apc_segment;
+
+/* Host-to-device upload executed by the SMs: the CTAs of one kernel load the
+ * sources in 16-byte words (bytes outside mutually 16-byte-aligned runs one
+ * by one) and store them to device memory.  On Grace-Blackwell the loads
+ * cross NVLink-C2C at the link's rate and need no DMA copy engine.  The
+ * kernel runs on at most max_ctas CTAs (0 = one per SM; 1 .. 4096), so that
+ * it can run on another stream beside this library's persistent kernels when
+ * those leave SMs free (apc_set_reserved_sms): for example, the next
+ * gradients' upload beside the current step.  Segments' destinations must
+ * not overlap.  bytes == 0 segments are skipped.  Ordered on `stream` like
+ * a kernel; the call never synchronizes.
+ * Returns APC_EINVAL (null pointers, num_segments < 0, max_ctas out of
+ * range, a source the device cannot read, a destination that is not device
+ * memory, overlapping destinations), APC_ERANGE (address + bytes overflows),
+ * APC_ECUDA, or APC_OK. */
+apc_status apc_upload(const apc_segment *segs, int32_t num_segments, int32_t max_ctas, apc_stream_t stream);
+
+/* Leave n SMs free of this library's persistent kernels: later launches of
+ * the step, digest and guard kernels run at most (SM count - n) x residency
+ * CTAs (at least one SM's worth), so that kernels of other streams, such as
+ * apc_upload, run beside them.  Results do not depend on it.  Process-wide,
+ * for every device; n: 0 (the default) .. 1024.  Returns APC_EINVAL for n
+ * out of range. */
+apc_status apc_set_reserved_sms(int32_t n);
+
 /* Device-side status of this library's kernels on the current device since
  * the previous call: APC_OK, or APC_ETIMEOUT if a bounded wait inside a
  * kernel gave up (the digests and updates of that launch are then incomplete;
@@ -217,7 +254,7 @@ const char *apc_status_string(apc_status s);
  * pointer stays valid until that thread's next apc_* call. */
 const char *apc_last_error(void);
 
-/* ABI version of this header: 2. */
+/* ABI version of this header: 3. */
 int32_t apc_version(void);
 
 #ifdef __cplusplus

@@ -15,6 +15,9 @@ Entry points mirror the C names:
   read only (post-recovery verification).
 * :func:`resolve_hparams` -> ``apc_resolve_hparams``: the step's binary32
   scalars (host only).
+* :func:`upload` -> ``apc_upload``: host-to-device upload executed by a
+  bounded number of CTAs, and :func:`set_reserved_sms` ->
+  ``apc_set_reserved_sms``: SMs the persistent kernels leave free for it.
 
 A table or buffer list that is used every step can be marshalled once with
 :func:`prepare_table` / :func:`prepare_buffers` and passed in its place.
@@ -30,7 +33,8 @@ from . import _build
 
 __all__ = ["TensorEntry", "TensorEntryBF16", "BufferEntry", "PreparedTable", "ApcError", "commit_step",
            "commit_step_bf16", "digest", "count_nonzero", "prepare_table", "prepare_buffers", "resolve_hparams",
-           "library", "lib_path", "F32", "BF16", "DEFAULT_HPARAMS"]
+           "Segment", "upload", "prepare_segments", "set_reserved_sms", "library", "lib_path", "F32", "BF16",
+           "DEFAULT_HPARAMS"]
 
 F32, BF16 = 0, 1
 MASK64 = (1 << 64) - 1
@@ -50,6 +54,10 @@ class _TensorBF16(ctypes.Structure):
 class _Buffer(ctypes.Structure):
     _fields_ = [("data", ctypes.c_void_p), ("n", ctypes.c_uint64), ("global_offset", ctypes.c_uint64),
                 ("dtype", ctypes.c_uint32), ("slot", ctypes.c_uint32)]
+
+
+class _Segment(ctypes.Structure):
+    _fields_ = [("dst", ctypes.c_void_p), ("src", ctypes.c_void_p), ("bytes", ctypes.c_uint64)]
 
 
 class _HParams(ctypes.Structure):
@@ -99,6 +107,10 @@ def library():
         lib.apc_device_status.restype = ctypes.c_int
         lib.apc_selftest_wait_timeout.argtypes = [ctypes.c_uint64, vp]
         lib.apc_selftest_wait_timeout.restype = ctypes.c_int
+        lib.apc_upload.argtypes = [vp, i32, i32, vp]
+        lib.apc_upload.restype = ctypes.c_int
+        lib.apc_set_reserved_sms.argtypes = [i32]
+        lib.apc_set_reserved_sms.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -333,6 +345,64 @@ def count_nonzero(buffers: Iterable[BufferEntry] | PreparedTable, num_slots: int
     _check(library().apc_count_nonzero(ctypes.addressof(arr), n, int(num_slots), ctypes.c_void_p(_stream(stream)),
                                        ctypes.c_void_p(_ptr(out, 8))))
     return out
+
+
+@dataclass
+class Segment:
+    """One upload segment: ``bytes`` bytes from ``src`` (a page-locked CPU
+    tensor, a CUDA tensor, or a raw pointer the device can read) to ``dst``
+    (a CUDA tensor or raw device pointer).  ``bytes`` defaults to dst's size."""
+    dst: object
+    src: object
+    bytes: int | None = None
+
+
+def _addr(x) -> int:
+    if isinstance(x, int):
+        return x
+    if not x.is_contiguous():
+        raise ValueError("tensor is not contiguous")
+    return x.data_ptr()
+
+
+def _segments(segments):
+    if isinstance(segments, PreparedTable):
+        if segments.kind != "segments":
+            raise ValueError("prepared table is a %s table, expected a segment list" % segments.kind)
+        return segments.arr, segments.count
+    segments = list(segments)
+    arr = (_Segment * max(1, len(segments)))()
+    for i, g in enumerate(segments):
+        n = g.bytes
+        if n is None:
+            n = g.dst.numel() * g.dst.element_size()
+        for name, t in (("dst", g.dst), ("src", g.src)):
+            if not isinstance(t, int) and t.numel() * t.element_size() < n:
+                raise ValueError("segments[%d].%s holds fewer than %d bytes" % (i, name, n))
+        if not isinstance(g.dst, int) and not g.dst.is_cuda:
+            raise ValueError("segments[%d].dst is not a CUDA tensor" % i)
+        arr[i] = _Segment(_addr(g.dst), _addr(g.src), int(n))
+    return arr, len(segments)
+
+
+def prepare_segments(segments: Iterable[Segment]) -> PreparedTable:
+    """Marshal an upload segment list once for :func:`upload`."""
+    segments = list(segments)
+    arr, n = _segments(segments)
+    return PreparedTable("segments", arr, n, None, segments)
+
+
+def upload(segments: Iterable[Segment] | PreparedTable, max_ctas: int = 0, stream=None) -> None:
+    """Enqueue the SM-driven host-to-device upload of ``segments`` on at
+    most ``max_ctas`` CTAs (``apc_upload``; 0 = one per SM)."""
+    arr, n = _segments(segments)
+    _check(library().apc_upload(ctypes.addressof(arr), n, int(max_ctas), ctypes.c_void_p(_stream(stream))))
+
+
+def set_reserved_sms(n: int) -> None:
+    """Leave ``n`` SMs free of the library's persistent kernels
+    (``apc_set_reserved_sms``; 0 restores the default)."""
+    _check(library().apc_set_reserved_sms(int(n)))
 
 
 def digests_to_host(out) -> list[int]:

@@ -21,7 +21,7 @@ LIB = os.path.join(BUILD, "libapc.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # exact IEEE binary32: no contraction into FMA, IEEE divide and sqrt, denormals kept
 NUMERIC = ["-fmad=false", "-prec-div=true", "-prec-sqrt=true", "-ftz=false"]
-UNITS = ["apc_commit.cu", "apc_digest.cu", "apc_guard.cu", "apc_host.cpp"]
+UNITS = ["apc_commit.cu", "apc_digest.cu", "apc_guard.cu", "apc_upload.cu", "apc_host.cpp"]
 
 
 def sources() -> list[str]:

@@ -125,10 +125,15 @@ apc_status device_info(Device *out) {
   return APC_OK;
 }
 
-// The persistent grid: one CTA per resident slot, capped by APC_GRID_LIMIT
-// (read at every call) when that is a positive integer.
+// SMs that the persistent kernels leave free (apc_set_reserved_sms).
+std::atomic<int> g_reserved_sms{0};
+
+// The persistent grid: one CTA per resident slot on the SMs not reserved
+// (at least one SM's worth), capped by APC_GRID_LIMIT (read at every call)
+// when that is a positive integer.
 unsigned grid_for(uint64_t tiles, int sms, int per_sm) {
-  uint64_t cap = (uint64_t)sms * (uint64_t)std::max(per_sm, 1);
+  const int avail = std::max(1, sms - g_reserved_sms.load(std::memory_order_relaxed));
+  uint64_t cap = (uint64_t)avail * (uint64_t)std::max(per_sm, 1);
   if (const char *lim = std::getenv("APC_GRID_LIMIT")) {
     char *end = nullptr;
     const unsigned long long v = std::strtoull(lim, &end, 10);
@@ -404,6 +409,120 @@ APC_EXPORT apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs
                                                apc::launch_count_large, "count kernel launch");
 }
 
+namespace {
+
+// The device-side address of a source the current device can read: device
+// or managed memory, page-locked host memory mapped for the device, or
+// pageable host memory where the device reads it through the host's page
+// tables.  Null if the device cannot read it.
+const void *device_readable(const void *p, bool pageable_ok) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();  // clear the error state of the failed query
+    return pageable_ok ? p : nullptr;
+  }
+  switch (a.type) {
+    case cudaMemoryTypeDevice:
+    case cudaMemoryTypeManaged:
+      return p;
+    case cudaMemoryTypeHost:
+      return a.devicePointer;
+    default:
+      return pageable_ok ? p : nullptr;
+  }
+}
+
+bool device_writable(void *p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+}  // namespace
+
+APC_EXPORT apc_status apc_upload(const apc_segment *segs, int32_t num_segments, int32_t max_ctas,
+                                 apc_stream_t stream) {
+  g_last_error[0] = 0;
+  if (num_segments < 0) return fail(APC_EINVAL, "num_segments %d < 0", num_segments);
+  if (num_segments > 0 && !segs) return fail(APC_EINVAL, "segments pointer is null");
+  if (max_ctas < 0 || max_ctas > 4096) return fail(APC_EINVAL, "max_ctas %d outside 0..4096", max_ctas);
+  std::vector<apc::UploadEntry> entries;
+  entries.reserve((size_t)num_segments);
+  int dev = 0, pageable = 0;
+  bool queried = false;
+  for (int32_t k = 0; k < num_segments; ++k) {
+    const apc_segment &g = segs[k];
+    if (g.bytes == 0) continue;
+    if (!g.dst || !g.src) return fail(APC_EINVAL, "segments[%d]: null pointer", k);
+    if (g.bytes > UINTPTR_MAX - (uintptr_t)g.dst || g.bytes > UINTPTR_MAX - (uintptr_t)g.src)
+      return fail(APC_ERANGE, "segments[%d]: address + bytes overflows", k);
+    if (!queried) {
+      int e = (int)cudaGetDevice(&dev);
+      if (e) return cuda_fail(e, "cudaGetDevice");
+      if ((e = (int)cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev)))
+        return cuda_fail(e, "cudaDeviceGetAttribute");
+      queried = true;
+    }
+    const void *src = device_readable(g.src, pageable != 0);
+    if (!src) return fail(APC_EINVAL, "segments[%d]: the device cannot read the source", k);
+    if (!device_writable(g.dst)) return fail(APC_EINVAL, "segments[%d]: destination is not device memory", k);
+    apc::UploadEntry e{};
+    e.dst = static_cast<uint8_t *>(g.dst);
+    e.src = static_cast<const uint8_t *>(src);
+    e.bytes = g.bytes;
+    const uintptr_t d = (uintptr_t)e.dst, s = (uintptr_t)e.src;
+    const uint64_t head = (16 - (d & 15)) & 15;
+    e.body = ((d ^ s) & 15) == 0 && g.bytes > head ? (g.bytes - head) & ~(uint64_t)15 : 0;
+    e.tile_begin = (e.body + apc::kUploadTile - 1) / apc::kUploadTile;  // tile count until placed
+    e.scalar_begin = g.bytes - e.body;                                  // scalar count until placed
+    entries.push_back(e);
+  }
+  // destinations must not overlap (sorted sweep)
+  std::vector<Range> rs;
+  rs.reserve(entries.size());
+  for (const auto &e : entries) rs.push_back(Range{(uintptr_t)e.dst, (uintptr_t)e.dst + e.bytes, true});
+  if (overlaps(rs)) return fail(APC_EINVAL, "destination ranges overlap");
+  if (entries.empty()) return APC_OK;
+  Device d;
+  apc_status st = device_info(&d);
+  if (st != APC_OK) return st;
+  const unsigned cap = max_ctas > 0 ? (unsigned)max_ctas : (unsigned)d.sms;
+  auto plan = std::make_unique<apc::UploadPlan<apc::kUploadMax>>();
+  size_t i = 0;
+  while (i < entries.size()) {
+    const size_t k = std::min(entries.size() - i, (size_t)apc::kUploadMax);
+    uint64_t tiles = 0, scalars = 0;
+    for (size_t j = 0; j < k; ++j) {
+      apc::UploadEntry e = entries[i + j];
+      const uint64_t t = e.tile_begin, c = e.scalar_begin;
+      e.tile_begin = tiles;
+      e.scalar_begin = scalars;
+      tiles += t;
+      scalars += c;
+      plan->e[j] = e;
+    }
+    plan->count = (uint32_t)k;
+    plan->total_tiles = tiles;
+    plan->total_scalar = scalars;
+    const uint64_t want = std::max<uint64_t>(tiles, (scalars + apc::kUploadThreads - 1) / apc::kUploadThreads);
+    const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(want, cap));
+    int e = apc::launch_upload(*plan, grid, stream);
+    if (e) return cuda_fail(e, "upload kernel launch");
+    i += k;
+  }
+  return APC_OK;
+}
+
+APC_EXPORT apc_status apc_set_reserved_sms(int32_t n) {
+  g_last_error[0] = 0;
+  if (n < 0 || n > 1024) return fail(APC_EINVAL, "reserved SMs %d outside 0..1024", n);
+  g_reserved_sms.store(n, std::memory_order_relaxed);
+  return APC_OK;
+}
+
 APC_EXPORT apc_status apc_device_status(void) {
   g_last_error[0] = 0;
   int e = (int)cudaDeviceSynchronize();
@@ -436,4 +555,4 @@ APC_EXPORT const char *apc_status_string(apc_status s) {
 
 APC_EXPORT const char *apc_last_error(void) { return g_last_error; }
 
-APC_EXPORT int32_t apc_version(void) { return 2; }
+APC_EXPORT int32_t apc_version(void) { return 3; }

@@ -126,6 +126,48 @@ constexpr int kDigestLarge = 1000;
 static_assert(sizeof(DigestEntry) == 32, "entry layout");
 static_assert(sizeof(DigestPlan<kDigestLarge>) <= 32764, "kernel parameter limit");
 
+// One segment of the upload kernel (48 bytes).  Where dst and src are
+// mutually 16-byte aligned, the `body` bytes from dst + head on are copied
+// in 16-byte words, in tiles of kUploadTile bytes; the head (fewer than 16
+// bytes before dst's 16-byte boundary) and the tail (body end to `bytes`)
+// are "scalar items", copied byte by byte after the tiles.  Mutually
+// misaligned segments have body = 0 and head = bytes.
+struct UploadEntry {
+  uint8_t *dst;
+  const uint8_t *src;   // device-side address of the source
+  uint64_t bytes;
+  uint64_t body;
+  uint64_t tile_begin;   // first tile of the segment (prefix over the launch)
+  uint64_t scalar_begin;  // first scalar item of the segment
+};
+// head = bytes before dst's 16-byte boundary, derived on the device:
+// (16 - dst % 16) % 16 when body > 0.
+
+template <int MAXE>
+struct UploadPlan {
+  uint64_t total_tiles;
+  uint64_t total_scalar;
+  uint32_t count;
+  uint32_t pad_;
+  UploadEntry e[MAXE];
+};
+
+#ifndef APC_UPLOAD_THREADS
+#define APC_UPLOAD_THREADS 512
+#endif
+#ifndef APC_UPLOAD_UNROLL
+#define APC_UPLOAD_UNROLL 8
+#endif
+constexpr int kUploadThreads = APC_UPLOAD_THREADS;
+constexpr int kUploadUnroll = APC_UPLOAD_UNROLL;                                       // 16-byte words per thread per tile
+constexpr uint64_t kUploadTile = (uint64_t)kUploadThreads * kUploadUnroll * 16;      // 64 KB
+constexpr int kUploadMax = 600;
+static_assert(sizeof(UploadEntry) == 48, "entry layout");
+static_assert(sizeof(UploadPlan<kUploadMax>) <= 32764, "kernel parameter limit");
+
+// Upload kernel (apc_upload.cu): the plan's segments, on `grid` CTAs.
+int launch_upload(const UploadPlan<kUploadMax> &plan, unsigned grid, void *stream);
+
 // Launch wrappers (apc_commit.cu, apc_digest.cu).  They return a cudaError_t
 // value and launch on `stream` with `grid` CTAs.
 int launch_commit_small(const CommitPlan<kCommitSmall> &plan, int layout, bool zero_grad, unsigned grid,

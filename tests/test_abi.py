@@ -25,11 +25,11 @@ def declared_functions():
 def test_exports_every_declared_function():
     names = declared_functions()
     assert set(names) >= {"apc_commit_step", "apc_digest", "apc_resolve_hparams", "apc_status_string",
-                          "apc_last_error", "apc_version"}
+                          "apc_last_error", "apc_version", "apc_upload", "apc_set_reserved_sms"}
     lib = ctypes.CDLL(apc.lib_path() if os.path.exists(apc.lib_path()) else apc._build.build())
     for n in names:
         assert hasattr(lib, n), n
-    assert apc.library().apc_version() == 2
+    assert apc.library().apc_version() == 3
 
 
 def test_status_strings():
@@ -214,3 +214,27 @@ def test_prepared_table_marshals_like_the_list():
     assert ei.value.status == 2
     with pytest.raises(ValueError):
         apc.commit_step(b, 1, stream=0, out=0x10000)
+
+
+class _S(ctypes.Structure):
+    _fields_ = [("dst", ctypes.c_void_p), ("src", ctypes.c_void_p), ("bytes", ctypes.c_uint64)]
+
+
+def test_upload_and_reserve_argument_checks():
+    lib = apc.library()
+
+    def up(segs, ctas=0):
+        arr = (_S * max(1, len(segs)))(*segs)
+        return lib.apc_upload(ctypes.addressof(arr), len(segs), ctas, None)
+
+    assert lib.apc_upload(None, 1, 0, None) == 1
+    assert lib.apc_upload(None, 0, 0, None) == 0                # nothing to do
+    assert up([_S(BASE, BASE + (1 << 30), 64)], ctas=-1) == 1
+    assert up([_S(BASE, BASE + (1 << 30), 64)], ctas=5000) == 1
+    assert up([_S(None, BASE, 64)]) == 1
+    assert up([_S(BASE, None, 64)]) == 1
+    assert up([_S(M64 - 10, BASE, 100)]) == 3                  # address + bytes overflows
+    assert up([_S(None, None, 0), _S(BASE, BASE, 0)]) == 0     # empty segments are skipped
+    assert lib.apc_set_reserved_sms(-1) == 1
+    assert lib.apc_set_reserved_sms(1025) == 1
+    assert lib.apc_set_reserved_sms(0) == 0
