@@ -1,6 +1,6 @@
 """In-tree build of libapc.so for sm_103a (nvcc, no cmake).
 
-The three translation units compile in parallel; the result lands in
+The translation units compile in parallel; the result lands in
 ``paper_2609_18178_gb300/_build/<machine>/libapc.so`` (git-ignored), next to
 the sources, so a GPU host builds its own copy for its own architecture.
 """
