@@ -210,9 +210,9 @@ def group_pieces(sizes: list[int], n_groups: int) -> list[list[int]]:
 
 def _replica_main(idx: int, n_rep: int, port: int, workload: str, flip: int, q) -> None:
     """One replica of a hybrid-sharding replication group on the current
-    GPU: commit its (identical) shard, then, in two rounds, verify and agree
-    with the other replicas; in round 2 one bit of replica `flip`'s HBM state
-    is flipped first through a host-side copy.  Spawned, so it builds its own
+    GPU: commit its (identical) shard, then verify and agree with the other
+    replicas twice; before the second agreement one bit of replica `flip`'s
+    HBM state is flipped through a host-side copy.  Spawned, so it builds its own
     CUDA context; replicas never wait on each other's kernels, only on the
     host control plane."""
     import datetime
@@ -247,7 +247,7 @@ def _replica_main(idx: int, n_rep: int, port: int, workload: str, flip: int, q) 
             entries.append(apc.TensorEntry(b["p"][sl], b["m"][sl], b["v"][sl], b["g"][sl], b["w"][sl], pc.goff))
             vbufs += apc.state_buffers(b["p"][sl], b["m"][sl], b["v"][sl], b["w"][sl], pc.goff)
         dc = apc.digests_to_host(apc.commit_step(entries, step, HP))
-        rounds = []
+        passes = []
         for r, flip_here in enumerate((False, idx == flip)):
             if flip_here:
                 word = bufs[0]["p"][12345:12346].view(torch.int32).cpu()
@@ -260,11 +260,11 @@ def _replica_main(idx: int, n_rep: int, port: int, workload: str, flip: int, q) 
             t1 = time.perf_counter()
             try:
                 ag = cohort.agree(dist, step, 1, dv, shard=0, group=grp)
-                rounds.append(("agreed", ["%016x" % d for d in ag.whole_digests], (t1 - t0) * 1e3,
+                passes.append(("agreed", ["%016x" % d for d in ag.whole_digests], (t1 - t0) * 1e3,
                                ag.seconds * 1e3))
             except cohort.CohortMismatch as e:
-                rounds.append(("mismatch", (e.what, e.ranks), (t1 - t0) * 1e3, (time.perf_counter() - t1) * 1e3))
-        q.put((idx, dc, rounds))
+                passes.append(("mismatch", (e.what, e.ranks), (t1 - t0) * 1e3, (time.perf_counter() - t1) * 1e3))
+        q.put((idx, dc, passes))
         dist.destroy_process_group()
     except Exception as e:  # reported, never hangs the parent
         q.put((idx, None, "error: %r" % (e,)))
@@ -297,14 +297,14 @@ def replica_check(n_rep: int = 4, workload: str = "c4", flip: int = 3, timeout_s
     if errors:
         return {"replicas": n_rep, "error": errors[0]}
     commit_equal = all(r[1] == res[0][1] for r in res)
-    ok_round = [r[2][0] for r in res]
-    flip_round = [r[2][1] for r in res]
+    clean_pass = [r[2][0] for r in res]
+    flip_pass = [r[2][1] for r in res]
     return {"replicas": n_rep, "workload": workload, "commit_digests_equal": commit_equal,
-            "round1_agreed": all(o[0] == "agreed" for o in ok_round),
-            "round2_flip_replica": flip,
-            "round2_detected_by_all": all(o[0] == "mismatch" for o in flip_round),
-            "round2_diagnosis": flip_round[0][1] if flip_round[0][0] == "mismatch" else None,
-            "verify_ms_max": max(o[2] for o in ok_round), "agree_ms_max": max(o[3] for o in ok_round),
+            "clean_agreed": all(o[0] == "agreed" for o in clean_pass),
+            "flipped_replica": flip,
+            "flip_detected_by_all": all(o[0] == "mismatch" for o in flip_pass),
+            "flip_diagnosis": flip_pass[0][1] if flip_pass[0][0] == "mismatch" else None,
+            "verify_ms_max": max(o[2] for o in clean_pass), "agree_ms_max": max(o[3] for o in clean_pass),
             "wall_s": time.perf_counter() - t0}
 
 

@@ -15,6 +15,6 @@ def test_two_replicas_agree_then_catch_a_flipped_bit():
     import bench
     r = bench.replica_check(2, "c3", flip=1, timeout_s=300)
     assert "error" not in r, r
-    assert r["commit_digests_equal"] and r["round1_agreed"]
-    assert r["round2_detected_by_all"]
-    assert tuple(r["round2_diagnosis"]) == ("state digests of shard 0", [0, 1])
+    assert r["commit_digests_equal"] and r["clean_agreed"]
+    assert r["flip_detected_by_all"]
+    assert tuple(r["flip_diagnosis"]) == ("state digests of shard 0", [0, 1])
