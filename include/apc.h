@@ -198,11 +198,12 @@ apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs, int32_t n
 apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t step, float out[8]);
 
 /* One segment of apc_upload: `bytes` bytes from `src` to `dst`.
- *   dst  device (or managed) memory of the current device, written
- *   src  memory the device can read: page-locked host memory mapped for the
- *        device (cudaHostAlloc, cudaHostRegister), pageable host memory on
- *        devices that read it through the host's page tables
- *        (cudaDevAttrPageableMemoryAccess), or device memory */
+ *   dst  device memory of the current device (or managed memory), written
+ *   src  memory the current device can read: page-locked host memory mapped
+ *        for the device (cudaHostAlloc, cudaHostRegister), pageable host
+ *        memory on devices that read it through the host's page tables
+ *        (cudaDevAttrPageableMemoryAccess), managed memory, or the current
+ *        device's own memory */
 typedef struct apc_segment {
   void *dst;
   const void *src;
@@ -216,13 +217,14 @@ typedef struct apc_segment {
  * kernel runs on at most max_ctas CTAs (0 = one per SM; 1 .. 4096), so that
  * it can run on another stream beside this library's persistent kernels when
  * those leave SMs free (apc_set_reserved_sms): for example, the next
- * gradients' upload beside the current step.  Segments' destinations must
- * not overlap.  bytes == 0 segments are skipped.  Ordered on `stream` like
+ * gradients' upload beside the current step.  A segment's destination must
+ * not overlap another destination or any source.  bytes == 0 segments are
+ * skipped.  Ordered on `stream` like
  * a kernel; the call never synchronizes.
  * Returns APC_EINVAL (null pointers, num_segments < 0, max_ctas out of
- * range, a source the device cannot read, a destination that is not device
- * memory, overlapping destinations), APC_ERANGE (address + bytes overflows),
- * APC_ECUDA, or APC_OK. */
+ * range, a source the current device cannot read, a destination outside the
+ * current device's memory, overlapping ranges), APC_ERANGE (address + bytes
+ * overflows), APC_ECUDA, or APC_OK. */
 apc_status apc_upload(const apc_segment *segs, int32_t num_segments, int32_t max_ctas, apc_stream_t stream);
 
 /* Leave n SMs free of this library's persistent kernels: later launches of

@@ -411,11 +411,11 @@ APC_EXPORT apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs
 
 namespace {
 
-// The device-side address of a source the current device can read: device
-// or managed memory, page-locked host memory mapped for the device, or
-// pageable host memory where the device reads it through the host's page
-// tables.  Null if the device cannot read it.
-const void *device_readable(const void *p, bool pageable_ok) {
+// The device-side address of a source the current device `dev` can read:
+// its own device memory, managed memory, page-locked host memory mapped for
+// the device, or pageable host memory where the device reads it through the
+// host's page tables.  Null if the device cannot read it.
+const void *device_readable(const void *p, int dev, bool pageable_ok) {
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
     cudaGetLastError();  // clear the error state of the failed query
@@ -423,6 +423,7 @@ const void *device_readable(const void *p, bool pageable_ok) {
   }
   switch (a.type) {
     case cudaMemoryTypeDevice:
+      return a.device == dev ? p : nullptr;
     case cudaMemoryTypeManaged:
       return p;
     case cudaMemoryTypeHost:
@@ -432,13 +433,14 @@ const void *device_readable(const void *p, bool pageable_ok) {
   }
 }
 
-bool device_writable(void *p) {
+// Device memory of `dev` (or managed memory) that a kernel may write.
+bool device_writable(void *p, int dev) {
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
     cudaGetLastError();
     return false;
   }
-  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+  return (a.type == cudaMemoryTypeDevice && a.device == dev) || a.type == cudaMemoryTypeManaged;
 }
 
 }  // namespace
@@ -466,9 +468,10 @@ APC_EXPORT apc_status apc_upload(const apc_segment *segs, int32_t num_segments, 
         return cuda_fail(e, "cudaDeviceGetAttribute");
       queried = true;
     }
-    const void *src = device_readable(g.src, pageable != 0);
-    if (!src) return fail(APC_EINVAL, "segments[%d]: the device cannot read the source", k);
-    if (!device_writable(g.dst)) return fail(APC_EINVAL, "segments[%d]: destination is not device memory", k);
+    const void *src = device_readable(g.src, dev, pageable != 0);
+    if (!src) return fail(APC_EINVAL, "segments[%d]: the current device cannot read the source", k);
+    if (!device_writable(g.dst, dev))
+      return fail(APC_EINVAL, "segments[%d]: destination is not memory of the current device", k);
     apc::UploadEntry e{};
     e.dst = static_cast<uint8_t *>(g.dst);
     e.src = static_cast<const uint8_t *>(src);
@@ -480,11 +483,14 @@ APC_EXPORT apc_status apc_upload(const apc_segment *segs, int32_t num_segments, 
     e.scalar_begin = g.bytes - e.body;                                  // scalar count until placed
     entries.push_back(e);
   }
-  // destinations must not overlap (sorted sweep)
+  // destinations must not overlap each other or any source (sorted sweep)
   std::vector<Range> rs;
-  rs.reserve(entries.size());
-  for (const auto &e : entries) rs.push_back(Range{(uintptr_t)e.dst, (uintptr_t)e.dst + e.bytes, true});
-  if (overlaps(rs)) return fail(APC_EINVAL, "destination ranges overlap");
+  rs.reserve(2 * entries.size());
+  for (const auto &e : entries) {
+    rs.push_back(Range{(uintptr_t)e.dst, (uintptr_t)e.dst + e.bytes, true});
+    rs.push_back(Range{(uintptr_t)e.src, (uintptr_t)e.src + e.bytes, false});
+  }
+  if (overlaps(rs)) return fail(APC_EINVAL, "a destination range overlaps another destination or a source");
   if (entries.empty()) return APC_OK;
   Device d;
   apc_status st = device_info(&d);

@@ -92,6 +92,9 @@ def test_rejected_destinations():
     with pytest.raises(apc.ApcError) as e:                     # overlapping destinations
         apc.upload([apc.Segment(d[0:], h, 100), apc.Segment(d[64:], h, 100)])
     assert e.value.status == 1
+    with pytest.raises(apc.ApcError) as e:                     # a source overlapping a destination
+        apc.upload([apc.Segment(d[0:], d[1000:], 100), apc.Segment(d[1050:], h, 100)])
+    assert e.value.status == 1
 
 
 @pytest.mark.parametrize("reserved", [16, 151, 1024])
