@@ -110,3 +110,62 @@ def test_reserved_sms_do_not_change_results(reserved):
         assert apc.digests_to_host(apc.digest(bufs, 4)) == dref
     finally:
         apc.set_reserved_sms(0)
+
+
+def test_upload_commit_digest_captured_in_one_graph():
+    """Upload of the gradient from pinned host memory, the step and the
+    verification digest, captured once as a CUDA graph; each replay uploads
+    the gradient the host wrote since, and the chained state equals the
+    oracle's."""
+    import synth
+    from test_gpu_parity import assert_same, dev, gen
+    specs = [(40_000, (1 << 32) - 20_000), (3, 300_000), (9_999, 300_003)]
+    tensors = [gen(n, off, 1) for n, off in specs]
+    devs, entries, hosts, segs = [], [], [], []
+    for t in tensors:
+        d = dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=torch.zeros(t["p"].size, dtype=torch.int16,
+                                                                            device="cuda"),
+                 w=torch.zeros(t["p"].size, dtype=torch.int16, device="cuda"))
+        devs.append(d)
+        entries.append(apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], t["goff"]))
+        h = torch.zeros(t["p"].size, dtype=torch.int16, pin_memory=True)
+        hosts.append(h)
+        segs.append(apc.Segment(d["g"], h))
+    vb = [b for e in entries for b in apc.state_buffers(e.p, e.m, e.v, e.w, e.global_offset)]
+    out_c = torch.empty(4, dtype=torch.int64, device="cuda")
+    out_v = torch.empty(4, dtype=torch.int64, device="cuda")
+    tab, vtab, seg = apc.prepare_table(entries), apc.prepare_buffers(vb), apc.prepare_segments(segs)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):                       # first calls outside capture (per-device queries)
+        apc.upload(seg, 4, stream=s)
+        apc.commit_step(tab, 7, stream=s, out=out_c)
+    torch.cuda.synchronize()
+    for t, d in zip(tensors, devs):                  # back to the generated state
+        for k in "pmv":
+            d[k].copy_(torch.from_numpy(t[k]).cuda())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(graph, stream=s):
+            apc.upload(seg, 4, stream=s)
+            apc.commit_step(tab, 7, stream=s, out=out_c)
+            apc.digest(vtab, 4, stream=s, out=out_v)
+    torch.cuda.synchronize()
+    for t, d in zip(tensors, devs):
+        for k in "pmv":
+            d[k].copy_(torch.from_numpy(t[k]).cuda())
+    h8 = oracle.resolve_hparams(oracle.DEFAULT_HP, 7)
+    ref = [dict(p=t["p"].copy(), m=t["m"].copy(), v=t["v"].copy(), goff=t["goff"]) for t in tensors]
+    for rep in range(3):                             # a new gradient from the host before every replay
+        for (n, off), h, r in zip(specs, hosts, ref):
+            g = synth.grad(n, off, 10 + rep)
+            h.copy_(torch.from_numpy(g.view(np.int16)))
+            r["g"] = g
+        graph.replay()
+        torch.cuda.synchronize()
+        ws, dref = oracle.commit_table(ref, h8)
+        for r, wv in zip(ref, ws):
+            r["w"] = wv
+        assert_same(devs, apc.digests_to_host(out_c), ref, dref)
+        assert apc.digests_to_host(out_v) == dref
+        for d, r in zip(devs, ref):
+            assert np.array_equal(d["g"].cpu().numpy().view(np.uint16), r["g"])
