@@ -22,11 +22,11 @@
 //    first digest index) into shared memory before arming the stage, so the
 //    consumers never search the chunk table themselves.
 //  * The consumer warps (19 by default) wait for a stage, read its
-//    descriptor and their elements from shared memory (thread t of C takes elements 4t..4t+3 and
-//    4C+4t..4C+4t+3, so both the shared-memory reads and the global stores
-//    are contiguous across the warp), release the stage to the producer, then
-//    apply AdamW, store the results with streaming stores, and fold the
-//    digest terms into 64-bit registers.
+//    descriptor and their elements from shared memory (thread t of C takes
+//    elements 4t..4t+3 and 4C+4t..4C+4t+3, so both the shared-memory reads
+//    and the global stores are contiguous across the warp), release the
+//    stage to the producer, then apply AdamW, store the results with
+//    streaming stores, and fold the digest terms into 64-bit registers.
 //  * Elements outside the aligned bodies (entry heads and tails under 8
 //    elements, and entries whose buffers are not mutually 16-byte aligned)
 //    are "scalar items", done afterwards by the consumers with a grid-stride

@@ -1,6 +1,8 @@
 // Host side of the C ABI declared in include/apc.h: argument validation,
 // resolution of the step's binary32 scalars (in double, rounded once),
-// conversion of the chunk table into launch plans, and the launches.
+// conversion of chunk tables, buffer lists and upload segments into launch
+// plans, the persistent grid sizes (SM count x residency, less the SMs
+// reserved with apc_set_reserved_sms), and the launches.
 //
 // The library allocates nothing.  Each plan travels in the kernel's
 // parameter block; the digests are accumulated with atomics straight into
