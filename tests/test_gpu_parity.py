@@ -676,3 +676,59 @@ def test_step_captured_in_a_cuda_graph_replays_bit_exact():
             r["w"] = wv
         assert_same(devs, apc.digests_to_host(out_c), ref, dref)
         assert apc.digests_to_host(out_v) == dref
+
+
+def test_concurrent_host_threads_on_separate_streams():
+    """Four host threads, each with its own stream and tables, call the
+    step and the digest repeatedly at the same time; every result equals
+    the oracle's (the library's per-device state and per-thread error
+    state are shared safely)."""
+    import threading
+    jobs = []
+    for j in range(4):
+        tensors = [gen(n, off, 2) for n, off in ((20_000 + 17 * j, (1 << 32) - 7_000 * (j + 1)), (9, 10 ** 6 * (j + 1)))]
+        devs = [dict(p=dev(t["p"]), m=dev(t["m"]), v=dev(t["v"]), g=dev(t["g"]),
+                     w=torch.zeros(t["p"].size, dtype=torch.int16, device="cuda")) for t in tensors]
+        jobs.append((tensors, devs))
+    torch.cuda.synchronize()
+    results, errors = [None] * 4, []
+
+    def work(j):
+        try:
+            tensors, devs = jobs[j]
+            s = torch.cuda.Stream()
+            entries = [apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], t["goff"]) for d, t in zip(devs, tensors)]
+            vb = [b for e in entries for b in apc.state_buffers(e.p, e.m, e.v, e.w, e.global_offset)]
+            got = []
+            for _ in range(5):                        # five chained steps, t = 2
+                with torch.cuda.stream(s):
+                    oc = apc.commit_step(entries, 2, HP, stream=s)
+                    ov = apc.digest(vb, 4, stream=s)
+                s.synchronize()
+                got.append((apc.digests_to_host(oc), apc.digests_to_host(ov)))
+            results[j] = got
+        except Exception as e:  # reported by the main thread
+            errors.append(repr(e))
+
+    threads = [threading.Thread(target=work, args=(j,)) for j in range(4)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors, errors
+    h8 = oracle.resolve_hparams(HP, 2)
+    for j, (tensors, devs) in enumerate(jobs):
+        ref = [dict(p=t["p"].copy(), m=t["m"].copy(), v=t["v"].copy(), g=t["g"], goff=t["goff"]) for t in tensors]
+        for k in range(5):
+            ws, dref = oracle.commit_table(ref, h8)
+            for r, wv in zip(ref, ws):
+                r["w"] = wv
+            assert results[j][k] == (dref, dref), (j, k)
+        assert_same(devs, dref, ref, dref)
+
+
+@pytest.mark.parametrize("value", ["", "abc", "0", "-5", "12x", "99999999999999999999"])
+def test_malformed_grid_limit_is_ignored(monkeypatch, value):
+    monkeypatch.setenv("APC_GRID_LIMIT", value)
+    tensors = [gen(n, off, 3) for n, off in ((50_001, 123), (6, 50_124))]
+    assert_same(*run_small(tensors, 3))
