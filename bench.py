@@ -44,6 +44,18 @@ FALLBACK_HBM_GBS = 6800.0
 
 # ----------------------------------------------------------------- helpers
 
+L2_BYTES = 129 << 20          # the GB300's L2
+
+# What each synthetic workload stands for (synth/workloads.py).
+WORKLOAD_TEXT = {
+    "c1": "one flat shard of 1,048,576 elements",
+    "c2": "one Mistral-7B MLP FSDP unit (gate, up, down) as one flat shard",
+    "c3": "ragged shard of a 1.216B-parameter decoder for 8 ranks",
+    "c4": "Mistral-7B rank shard 9 of 16, crossing tensor boundaries",
+    "c5": "full Mistral-7B shard on one GPU",
+}
+
+
 def measured_peak():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -579,6 +591,8 @@ def run_gpu(args):
             dist.destroy_process_group()
         return
     peak, peak_kind = measured_peak()
+    n_commit_launches = max(1, (len(entries) + 439) // 440)
+    n_digest_launches = max(1, (len(vbufs) + 999) // 1000)
     c_ms = statistics.median(commit_ms)
     v_ms = statistics.median(verify_ms)
     c_avg = sum(commit_ms) / K
@@ -596,10 +610,13 @@ def run_gpu(args):
         "vs_baseline": None,
         "dtype": "f32+u64",
         "data": "synthetic",
-        "config": {"workload": "%s: full Mistral-7B shard on one GPU, %d tensors, %d elements, step %d, "
-                               "commit+digest then re-verify" % (w.name, len(w.pieces), N, step_t),
-                   "elements": N, "tensors": len(w.pieces), "step": step_t, "parallelism": "%d ranks x one shard each (no data-path collective)" % world,
-                   "l2": "inputs larger than L2 (%.0f GB resident state)" % (16 * N / 1e9)},
+        "config": {"workload": "%s: %s, %d tensors, %d elements, step %d, commit+digest then re-verify"
+                               % (w.name, WORKLOAD_TEXT.get(w.name, "synthetic shard"), len(w.pieces), N, step_t),
+                   "elements": N, "tensors": len(w.pieces), "step": step_t,
+                   "parallelism": "%d ranks x one shard each (no data-path collective)" % world,
+                   "l2": ("inputs larger than L2 (%.1f GB resident state)" % (16 * N / 1e9)
+                          if COMMIT_BYTES * N > L2_BYTES else
+                          "inputs smaller than L2 (%.3f GB per step): timings include L2 hits" % (COMMIT_BYTES * N / 1e9))},
         "hbm_gbs_step": (COMMIT_BYTES + VERIFY_BYTES) * N / (ms_per_step * 1e-3) / 1e9,
         "commit_ms": c_ms,
         "verify_ms": v_ms,
@@ -611,8 +628,10 @@ def run_gpu(args):
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": profiled_traffic("commit_kernel", w.name),
                      "algorithmic_bytes_per_launch": COMMIT_BYTES * N},
-        "gpu_launches": K * (1 + (len(vbufs) + 999) // 1000),
-        "gpu_launches_note": "per timed step: 1 commit_kernel + 2 digest_kernel launches (1164 buffers, 1000 per launch)",
+        "gpu_launches": K * (n_commit_launches + n_digest_launches),
+        "gpu_launches_note": "per timed step: %d commit_kernel + %d digest_kernel launches (%d tensors, %d buffers; "
+                             "up to 440 tensors and 1000 buffers per launch)"
+                             % (n_commit_launches, n_digest_launches, len(entries), len(vbufs)),
         "digests": ["%016x" % d for d in whole],
         "verify_matches_commit": verified,
         "clocks": clk,
