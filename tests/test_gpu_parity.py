@@ -732,3 +732,34 @@ def test_malformed_grid_limit_is_ignored(monkeypatch, value):
     monkeypatch.setenv("APC_GRID_LIMIT", value)
     tensors = [gen(n, off, 3) for n, off in ((50_001, 123), (6, 50_124))]
     assert_same(*run_small(tensors, 3))
+
+
+def test_bf16_copy_of_every_binary32_pattern():
+    """With lr = 0 and m = v = g = 0 the step leaves p' = p exactly, so w is
+    the kernel's bf16 rounding of p itself.  Every one of the 2^32 bit
+    patterns (NaNs excepted: outside the contract) goes through the commit
+    kernel in chunks of 2^28; p' and w equal the oracle's bit for bit."""
+    hp = dict(HP, lr=0.0)
+    chunk = 1 << 28
+    p = torch.empty(chunk, dtype=torch.int32, device="cuda")
+    m = torch.zeros(chunk, dtype=torch.float32, device="cuda")
+    v = torch.zeros(chunk, dtype=torch.float32, device="cuda")
+    g = torch.zeros(chunk, dtype=torch.int16, device="cuda")
+    w = torch.empty(chunk, dtype=torch.int16, device="cuda")
+    tab = apc.prepare_table([apc.TensorEntry(p, m, v, g, w, 0)])
+    base = np.arange(chunk, dtype=np.uint32)
+    u = np.empty_like(base)
+    for start in range(0, 1 << 32, chunk):
+        p.copy_(torch.arange(start, start + chunk, dtype=torch.int64, device="cuda").to(torch.int32))
+        m.zero_()
+        v.zero_()
+        apc.commit_step(tab, 1, hp)
+        np.add(base, np.uint32(start), out=u)
+        f = u.view(np.float32)
+        keep = ~np.isnan(f)
+        got_p = p.cpu().numpy().view(np.uint32)
+        got_w = w.cpu().numpy().view(np.uint16)
+        assert np.array_equal(got_p[keep], u[keep]), hex(start)
+        assert np.array_equal(got_w[keep], oracle.bf16_rne(f)[keep]), hex(start)
+    del p, m, v, g, w
+    torch.cuda.empty_cache()
