@@ -411,12 +411,22 @@ def run_gpu(args):
     # kernels leave free (apc_set_reserved_sms); --e2e-upload copy uses the
     # DMA copy engines (cudaMemcpyAsync per tensor) instead.
     e2e = None
+    host_g = []
     if not args.no_e2e:
-        host_g = []
-        for b in bufs:
-            hg = torch.empty(b["g"].numel(), dtype=torch.int16, pin_memory=True)
-            hg.copy_(b["g"])
-            host_g.append(hg)
+        # every rank pins its own copy of the gradient; the leg runs only if
+        # all ranks could (a rank without it would leave the others waiting)
+        why = ""
+        try:
+            for b in bufs:
+                hg = torch.empty(b["g"].numel(), dtype=torch.int16, pin_memory=True)
+                hg.copy_(b["g"])
+                host_g.append(hg)
+        except RuntimeError as ex:
+            host_g, why = [], (str(ex).splitlines() or [type(ex).__name__])[0]
+        if max_over_ranks(dist, 0.0 if why == "" else 1.0) > 0:
+            e2e = {"error": "pinned host memory for the gradient (%.1f GB per rank) could not be allocated on "
+                            "every rank%s" % (2 * N / 1e9, ": " + why if why else "")}
+    if not args.no_e2e and e2e is None:
         groups = group_pieces([pc.n for pc in w.pieces], args.e2e_groups)
         n_groups = len(groups)
         copy_stream = torch.cuda.Stream(device=dev)
