@@ -65,13 +65,21 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash() -> str:
-    """Hash of the kernel sources' code (comments and blank space removed), so
-    that the recorded ncu traffic is dropped whenever the code changes."""
+# The sources each profiled kernel is compiled from (its translation unit and
+# the device headers it includes); host code only launches it.
+KERNEL_SOURCES = {
+    "commit_kernel": ["apc_commit.cu", "apc_device.cuh", "apc_tma.cuh", "apc_internal.h"],
+    "digest_kernel": ["apc_digest.cu", "apc_device.cuh", "apc_internal.h"],
+}
+
+
+def kernel_source_hash(kernel: str) -> str:
+    """Hash of a kernel's sources with comments and blank space removed, so
+    that its recorded ncu traffic is dropped whenever its code changes."""
     import re
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_18178_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
+    for name in KERNEL_SOURCES[kernel]:
         with open(os.path.join(csrc, name)) as f:
             code = f.read()
         code = re.sub(r"/\*.*?\*/", " ", code, flags=re.S)
@@ -90,7 +98,7 @@ def profiled_traffic(kernel: str, workload: str):
             rec = json.load(f)[kernel]
     except (OSError, KeyError, ValueError):
         return None
-    if rec.get("source_hash") != kernel_source_hash():
+    if rec.get("source_hash") != kernel_source_hash(kernel):
         return None
     if rec.get("workload") != workload:
         return None
