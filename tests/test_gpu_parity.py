@@ -737,8 +737,12 @@ def test_malformed_grid_limit_is_ignored(monkeypatch, value):
 def test_bf16_copy_of_every_binary32_pattern():
     """With lr = 0 and m = v = g = 0 the step leaves p' = p exactly, so w is
     the kernel's bf16 rounding of p itself.  Every one of the 2^32 bit
-    patterns (NaNs excepted: outside the contract) goes through the commit
-    kernel in chunks of 2^28; p' and w equal the oracle's bit for bit."""
+    patterns goes through the commit kernel in chunks of 2^28: p' and w
+    equal the oracle's bit for bit (NaNs excepted: outside the contract),
+    and the fused digests of p', m', v', w equal the oracle's (chunks with
+    NaNs excepted), which pins the commit kernel's own splitmix64 form on
+    every low word."""
+    from concurrent.futures import ThreadPoolExecutor
     hp = dict(HP, lr=0.0)
     chunk = 1 << 28
     p = torch.empty(chunk, dtype=torch.int32, device="cuda")
@@ -746,14 +750,23 @@ def test_bf16_copy_of_every_binary32_pattern():
     v = torch.zeros(chunk, dtype=torch.float32, device="cuda")
     g = torch.zeros(chunk, dtype=torch.int16, device="cuda")
     w = torch.empty(chunk, dtype=torch.int16, device="cuda")
+    out = torch.empty(4, dtype=torch.int64, device="cuda")
     tab = apc.prepare_table([apc.TensorEntry(p, m, v, g, w, 0)])
     base = np.arange(chunk, dtype=np.uint32)
     u = np.empty_like(base)
+    zero_digest = oracle.digest_f32(np.zeros(chunk, dtype=np.uint32), 0)
+
+    def expected(start):
+        a = base + np.uint32(start)
+        return oracle.digest_f32(a, 0), oracle.digest_u16(oracle.bf16_rne(a.view(np.float32)), 0)
+
+    pool = ThreadPoolExecutor(4)
+    pending = []
     for start in range(0, 1 << 32, chunk):
         p.copy_(torch.arange(start, start + chunk, dtype=torch.int64, device="cuda").to(torch.int32))
         m.zero_()
         v.zero_()
-        apc.commit_step(tab, 1, hp)
+        d = apc.digests_to_host(apc.commit_step(tab, 1, hp, out=out))
         np.add(base, np.uint32(start), out=u)
         f = u.view(np.float32)
         keep = ~np.isnan(f)
@@ -761,5 +774,38 @@ def test_bf16_copy_of_every_binary32_pattern():
         got_w = w.cpu().numpy().view(np.uint16)
         assert np.array_equal(got_p[keep], u[keep]), hex(start)
         assert np.array_equal(got_w[keep], oracle.bf16_rne(f)[keep]), hex(start)
+        assert d[1] == zero_digest and d[2] == zero_digest, hex(start)
+        if keep.all():
+            pending.append((start, d, pool.submit(expected, start)))
+    for start, d, fut in pending:
+        dp, dw = fut.result()
+        assert d[0] == dp and d[3] == dw, hex(start)
+    pool.shutdown()
+    assert len(pending) == 14                     # the two chunks holding NaN patterns are left out
     del p, m, v, g, w
+    torch.cuda.empty_cache()
+
+
+def test_digest_of_every_low_word():
+    """A buffer whose element i holds bits i (i < 2^32), digested at global
+    offset 0 in chunks of 2^28: the keys (i << 32) | i cover every low word
+    and every index mod 2^32 once.  The wrapping sum of the GPU's chunk
+    digests equals the oracle's (digest concatenation)."""
+    from concurrent.futures import ThreadPoolExecutor
+    chunk = 1 << 28
+    starts = list(range(0, 1 << 32, chunk))
+    buf = torch.empty(chunk, dtype=torch.int32, device="cuda")
+    out = torch.empty(1, dtype=torch.int64, device="cuda")
+    got = 0
+    for start in starts:
+        buf.copy_(torch.arange(start, start + chunk, dtype=torch.int64, device="cuda").to(torch.int32))
+        got = (got + apc.digests_to_host(apc.digest([apc.BufferEntry(buf, 0, start, apc.F32)], 1, out=out))[0]) & M64
+
+    def part(start):
+        return oracle.digest_f32(np.arange(chunk, dtype=np.uint32) + np.uint32(start), start)
+
+    with ThreadPoolExecutor(4) as ex:
+        want = sum(ex.map(part, starts)) & M64
+    assert got == want
+    del buf
     torch.cuda.empty_cache()
