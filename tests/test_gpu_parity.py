@@ -809,3 +809,88 @@ def test_digest_of_every_low_word():
     assert got == want
     del buf
     torch.cuda.empty_cache()
+
+
+def test_every_bf16_parameter_and_gradient_pair():
+    """Every pair (p, g) of a bf16 bit pattern p (widened to binary32) and a
+    bf16 gradient g, 2^32 elements at m = v = 0, through the fp32 commit
+    kernel in chunks of 2^28; NaN parameters and non-finite gradients, which
+    are outside the contract, are replaced by +0.  p', m', v', w and the
+    four digests equal the oracle's bit for bit."""
+    import os
+    chunk = 1 << 28
+    nthreads = os.cpu_count() or 1
+    step = 3
+    h8 = oracle.resolve_hparams(HP, step)
+    idx = np.arange(chunk, dtype=np.uint32)
+    d = {k: torch.empty(chunk, dtype=torch.float32, device="cuda") for k in "pmv"}
+    d["g"] = torch.empty(chunk, dtype=torch.int16, device="cuda")
+    d["w"] = torch.empty(chunk, dtype=torch.int16, device="cuda")
+    out = torch.empty(4, dtype=torch.int64, device="cuda")
+    tab = apc.prepare_table([apc.TensorEntry(d["p"], d["m"], d["v"], d["g"], d["w"], 0)])
+    for start in range(0, 1 << 32, chunk):
+        i = idx + np.uint32(start)
+        p16 = (i >> 16).astype(np.uint16)
+        g16 = (i & 0xFFFF).astype(np.uint16)
+        p16[(p16 & 0x7FFF) > 0x7F80] = 0                     # NaN parameters
+        g16[(g16 & 0x7FFF) >= 0x7F80] = 0                    # infinite and NaN gradients
+        p = (p16.astype(np.uint32) << 16).view(np.float32)
+        m = np.zeros(chunk, dtype=np.float32)
+        v = np.zeros(chunk, dtype=np.float32)
+        d["p"].copy_(torch.from_numpy(p))
+        d["m"].zero_()
+        d["v"].zero_()
+        d["g"].copy_(torch.from_numpy(g16.view(np.int16)))
+        got = apc.digests_to_host(apc.commit_step(tab, step, HP, out=out))
+        w, dref = oracle.commit(p, m, v, g16, 0, h8, nthreads=nthreads)
+        for k, ref in (("p", p), ("m", m), ("v", v)):
+            a = d[k].cpu().numpy().view(np.uint32)
+            bad = np.nonzero(a != ref.view(np.uint32))[0]
+            assert bad.size == 0, (hex(start), k, bad[:4])
+        assert np.array_equal(d["w"].cpu().numpy().view(np.uint16), w), hex(start)
+        assert got == dref, hex(start)
+    del d
+    torch.cuda.empty_cache()
+
+
+def test_every_bf16_state_parameter_and_gradient_pair():
+    """The bf16-state step (the paper's precision) over every pair (p, g) of
+    bf16 bit patterns, 2^32 elements at m = v = 0, in chunks of 2^28; NaN
+    parameters and non-finite gradients are replaced by +0.  p', m', v' and
+    the three digests equal the oracle's bit for bit."""
+    import os
+    from concurrent.futures import ThreadPoolExecutor
+    chunk, sub = 1 << 28, 1 << 24
+    step = 3
+    h8 = oracle.resolve_hparams(HP, step)
+    idx = np.arange(chunk, dtype=np.uint32)
+    d = {k: torch.empty(chunk, dtype=torch.int16, device="cuda") for k in "pmvg"}
+    out = torch.empty(3, dtype=torch.int64, device="cuda")
+    tab = apc.prepare_table([apc.TensorEntryBF16(d["p"], d["m"], d["v"], d["g"], 0)])
+    pool = ThreadPoolExecutor(os.cpu_count() or 1)
+    for start in range(0, 1 << 32, chunk):
+        i = idx + np.uint32(start)
+        p = (i >> 16).astype(np.uint16)
+        g = (i & 0xFFFF).astype(np.uint16)
+        p[(p & 0x7FFF) > 0x7F80] = 0                          # NaN parameters
+        g[(g & 0x7FFF) >= 0x7F80] = 0                         # infinite and NaN gradients
+        m = np.zeros(chunk, dtype=np.uint16)
+        v = np.zeros(chunk, dtype=np.uint16)
+        d["p"].copy_(torch.from_numpy(p.view(np.int16)))
+        d["m"].zero_()
+        d["v"].zero_()
+        d["g"].copy_(torch.from_numpy(g.view(np.int16)))
+        got = apc.digests_to_host(apc.commit_step_bf16(tab, step, HP, out=out))
+        parts = pool.map(lambda s: oracle.commit_bf16(p[s:s + sub], m[s:s + sub], v[s:s + sub], g[s:s + sub], s, h8),
+                         range(0, chunk, sub))
+        want = [0, 0, 0]
+        for dd in parts:
+            want = [(a + b) & M64 for a, b in zip(want, dd)]
+        for k, ref in (("p", p), ("m", m), ("v", v)):
+            a = d[k].cpu().numpy().view(np.uint16)
+            bad = np.nonzero(a != ref)[0]
+            assert bad.size == 0, (hex(start), k, bad[:4])
+        assert got == want, hex(start)
+    pool.shutdown()
+    del d
+    torch.cuda.empty_cache()
