@@ -146,8 +146,10 @@ def textbook_adamw_double(p, m, v, G, t, hp=HP):
     step = lr / (1 - b1 ** t)
     bound_m = 3.1 * EPS32 * A
     bound_v = 3.1 * EPS32 * v1
+    # subnormal m' carries an absolute rounding error (up to 2^-150 per operation) that the division by den
+    # carries into u, hence the step * 2^-149 / den term
     bound_p = 1.25 * EPS32 * (2 * np.abs(p * (1 - lr * wd)) + step * (8.6 * np.abs(u) + 3.1 * A / den)
-                              + np.abs(p1)) + 2.0 ** -146
+                              + np.abs(p1)) + 1.25 * step * 2.0 ** -149 / den + 2.0 ** -146
     return p1, m1, v1, bound_p, bound_m, bound_v
 
 
@@ -179,6 +181,49 @@ def test_against_textbook_double_within_rounding_bound(t):
     assert np.all(np.abs(m - m1) <= bm + 2.0 ** -149), "m' outside the rounding bound"
     assert np.all(np.abs(v - v1) <= bv + 2.0 ** -149), "v' outside the rounding bound"
     assert np.all(np.abs(p - p1) <= bp), "p' outside the rounding bound"
+
+
+def every_gradient_state(g_all):
+    """Each gradient of g_all at five moment states and six parameter magnitudes."""
+    states = [(0.0, 0.0), (1e-4, 1e-6), (-3e-2, 4e-5), (1e-38, 1e-41), (2.5, 7.0)]
+    params = [0.0, 1e-30, -0.02, 0.7, -3.0e4, 1.0e30]
+    g = np.tile(g_all, len(states) * len(params))
+    m = np.repeat(np.array([s[0] for s in states], dtype=np.float32), g_all.size * len(params))
+    v = np.repeat(np.array([s[1] for s in states], dtype=np.float32), g_all.size * len(params))
+    p = np.tile(np.repeat(np.array(params, dtype=np.float32), g_all.size), len(states))
+    return p, m, v, g
+
+
+@pytest.mark.parametrize("t", [1, 18])
+def test_every_bf16_gradient_within_rounding_bound(t):
+    """Every bf16 gradient whose square is finite in binary32 (|g| < 2^64,
+    subnormals included) against the textbook update in double, at five
+    moment states and six parameter magnitudes each (1.5 million elements)."""
+    g_all = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)
+    g_all = g_all[(g_all & 0x7FFF) < 0x5F80]
+    p, m, v, g = every_gradient_state(g_all)
+    p1, m1, v1, bp, bm, bv = textbook_adamw_double(p, m, v, gf32(g), t)
+    oracle.adamw(p, m, v, g, oracle.resolve_hparams(HP, t))
+    assert np.all(np.abs(m - m1) <= bm + 2.0 ** -149), "m' outside the rounding bound"
+    assert np.all(np.abs(v - v1) <= bv + 2.0 ** -149), "v' outside the rounding bound"
+    assert np.all(np.abs(p - p1) <= bp), "p' outside the rounding bound"
+
+
+def test_gradients_whose_square_overflows():
+    """For finite |g| >= 2^64 the binary32 g*g overflows (IEEE: +inf), so
+    v' = +inf, den = +inf, u = m'/den = 0 and p' = p*(1 - lr*wd) exactly,
+    while m' stays finite and within its bound."""
+    g_all = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)
+    g_all = g_all[((g_all & 0x7FFF) >= 0x5F80) & ((g_all & 0x7FFF) < 0x7F80)]
+    p, m, v, g = every_gradient_state(g_all)
+    h = oracle.resolve_hparams(HP, 5)
+    decay = np.float32(h[5])
+    p_dec = p * decay
+    _, m1, _, _, bm, _ = textbook_adamw_double(p, m, v, gf32(g), 5)
+    oracle.adamw(p, m, v, g, h)
+    assert np.all(np.isposinf(v))
+    assert np.array_equal(p.view(np.uint32), p_dec.view(np.uint32))
+    assert np.all(np.abs(m - m1) <= bm + 2.0 ** -149)
 
 
 def test_bounds_would_catch_plausible_mistakes():
