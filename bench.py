@@ -563,6 +563,9 @@ def run_gpu(args):
         torch.cuda.synchronize()
         # f3: the paper's bf16-state rank shard (rank 1 of 4), committed and verified
         w3 = W.f3()
+        if args.f3_tensors:    # the first K tensors only (a smaller case for profiling)
+            kept = w3.pieces[:args.f3_tensors]
+            w3 = W.Workload(w3.name, kept, w3.steps, w3.chained, w3.verify, [max(pc.at + pc.n for pc in kept)])
         N3 = w3.n
         b3 = {k: torch.empty(N3, dtype=torch.int16, device=dev) for k in "pmvg"}
         g3 = w3.pieces[0].goff - w3.pieces[0].at
@@ -581,8 +584,8 @@ def run_gpu(args):
         f3v_ms = timed(lambda: apc.digest(v3, 3, stream=s, out=out3v), max(3, K))
         f3_ok = apc.digests_to_host(out3) == apc.digests_to_host(out3v)
         del b3, e3, v3
-        nxt = {"f3_commit_bf16_state": {"workload": "rank 1 of 4 of Mistral-7B, %d elements, 77 pieces, bf16 p/m/v"
-                                                    % N3, "ms": f3_ms, "gbs": 14 * N3 / (f3_ms * 1e-3) / 1e9,
+        nxt = {"f3_commit_bf16_state": {"workload": "rank 1 of 4 of Mistral-7B, %d elements, %d pieces, bf16 p/m/v"
+                                                    % (N3, len(w3.pieces)), "ms": f3_ms, "gbs": 14 * N3 / (f3_ms * 1e-3) / 1e9,
                                         "frac": 14 * N3 / (f3_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 14,
                                         "verify_ms": f3v_ms, "verify_gbs": 6 * N3 / (f3v_ms * 1e-3) / 1e9,
                                         "verify_matches_commit": f3_ok},
@@ -741,6 +744,8 @@ def main(argv=None):
     ap.add_argument("--workload", choices=["c1", "c2", "c3", "c4", "c5"], default="c5")
     ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--e2e-groups", type=int, default=12)
+    ap.add_argument("--f3-tensors", type=int, default=0,
+                    help="next row f3 over the first K tensors of its shard only (0 = all; for profiling)")
     ap.add_argument("--e2e-upload", choices=["sm", "copy"], default="sm",
                     help="end-to-end upload: apc_upload on a few CTAs, or the DMA copy engines")
     ap.add_argument("--e2e-upload-ctas", type=int, default=16)
