@@ -238,3 +238,33 @@ def test_upload_and_reserve_argument_checks():
     assert lib.apc_set_reserved_sms(-1) == 1
     assert lib.apc_set_reserved_sms(1025) == 1
     assert lib.apc_set_reserved_sms(0) == 0
+
+
+def test_last_error_is_per_thread():
+    """Threads that fail validation in different ways at the same time each
+    read back their own error detail (apc_last_error is thread-local)."""
+    import threading
+    lib = apc.library()
+    cases = [
+        (lambda: commit([fake(8)], step=0), 1, b"step"),
+        (lambda: commit([fake(8, p=2)]), 2, b"aligned"),
+        (lambda: commit([fake(100, goff=M64 - 50)]), 3, b"overflow"),
+        (lambda: lib.apc_set_reserved_sms(-3), 1, b"reserved"),
+    ]
+    failures = []
+
+    def run(k):
+        call, status, word = cases[k % len(cases)]
+        for _ in range(200):
+            st = call()
+            msg = lib.apc_last_error()
+            if st != status or word not in msg.lower():
+                failures.append((k, st, msg))
+                return
+
+    threads = [threading.Thread(target=run, args=(k,)) for k in range(8)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not failures, failures[:3]
