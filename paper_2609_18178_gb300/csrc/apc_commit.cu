@@ -90,6 +90,15 @@ struct __align__(16) StageDesc {
 };
 static_assert(sizeof(StageDesc) == 48, "three 16-byte shared-memory loads");
 
+// A commit digest term.  With SHARED the caller has established that the
+// whole group's terms share the top two bits of their incremented key high
+// word (top_bits_shared) and passes them as `top`.
+template <uint32_t K, bool SHARED>
+__device__ __forceinline__ uint64_t cterm(uint32_t G, uint32_t bits, uint32_t one, uint32_t top) {
+  if constexpr (SHARED) return digest_term<K>(G, bits, one, top);
+  else return digest_term<K>(G, bits, one);
+}
+
 // ------------------------------------------------------------ fp32 state
 
 struct F32State {
@@ -123,14 +132,29 @@ struct F32State {
     __stcs(reinterpret_cast<float4 *>(static_cast<float *>(d.m) + off), make_float4(m[0], m[1], m[2], m[3]));
     __stcs(reinterpret_cast<float4 *>(static_cast<float *>(d.v) + off), make_float4(v[0], v[1], v[2], v[3]));
     __stcs(reinterpret_cast<uint2 *>(d.w + off), make_uint2(w[0] | (w[1] << 16), w[2] | (w[3] << 16)));
-    a.p += digest_term<OFF>(G, __float_as_uint(p[0]), s.one) + digest_term<OFF + 1>(G, __float_as_uint(p[1]), s.one);
-    a.p += digest_term<OFF + 2>(G, __float_as_uint(p[2]), s.one) + digest_term<OFF + 3>(G, __float_as_uint(p[3]), s.one);
-    a.m += digest_term<OFF>(G, __float_as_uint(m[0]), s.one) + digest_term<OFF + 1>(G, __float_as_uint(m[1]), s.one);
-    a.m += digest_term<OFF + 2>(G, __float_as_uint(m[2]), s.one) + digest_term<OFF + 3>(G, __float_as_uint(m[3]), s.one);
-    a.v += digest_term<OFF>(G, __float_as_uint(v[0]), s.one) + digest_term<OFF + 1>(G, __float_as_uint(v[1]), s.one);
-    a.v += digest_term<OFF + 2>(G, __float_as_uint(v[2]), s.one) + digest_term<OFF + 3>(G, __float_as_uint(v[3]), s.one);
-    a.w += digest_term<OFF>(G, w[0], s.one) + digest_term<OFF + 1>(G, w[1], s.one);
-    a.w += digest_term<OFF + 2>(G, w[2], s.one) + digest_term<OFF + 3>(G, w[3], s.one);
+    // the group's keys are G + OFF .. G + OFF + 3
+    const uint32_t B = G + (0x9E3779B9u + OFF);
+    const uint32_t pb[4] = {__float_as_uint(p[0]), __float_as_uint(p[1]), __float_as_uint(p[2]), __float_as_uint(p[3])};
+    const uint32_t mb[4] = {__float_as_uint(m[0]), __float_as_uint(m[1]), __float_as_uint(m[2]), __float_as_uint(m[3])};
+    const uint32_t vb[4] = {__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]), __float_as_uint(v[3])};
+    if (top_bits_shared(B, 4)) {
+      fold<OFF, true>(G, pb, mb, vb, w, s.one, B >> 30, a);
+    } else {
+      fold<OFF, false>(G, pb, mb, vb, w, s.one, 0, a);
+    }
+  }
+
+  template <uint32_t OFF, bool SHARED>
+  __device__ static void fold(uint32_t G, const uint32_t (&p)[4], const uint32_t (&m)[4], const uint32_t (&v)[4],
+                              const uint32_t (&w)[4], uint32_t one, uint32_t top, Acc &a) {
+    a.p += cterm<OFF, SHARED>(G, p[0], one, top) + cterm<OFF + 1, SHARED>(G, p[1], one, top);
+    a.p += cterm<OFF + 2, SHARED>(G, p[2], one, top) + cterm<OFF + 3, SHARED>(G, p[3], one, top);
+    a.m += cterm<OFF, SHARED>(G, m[0], one, top) + cterm<OFF + 1, SHARED>(G, m[1], one, top);
+    a.m += cterm<OFF + 2, SHARED>(G, m[2], one, top) + cterm<OFF + 3, SHARED>(G, m[3], one, top);
+    a.v += cterm<OFF, SHARED>(G, v[0], one, top) + cterm<OFF + 1, SHARED>(G, v[1], one, top);
+    a.v += cterm<OFF + 2, SHARED>(G, v[2], one, top) + cterm<OFF + 3, SHARED>(G, v[3], one, top);
+    a.w += cterm<OFF, SHARED>(G, w[0], one, top) + cterm<OFF + 1, SHARED>(G, w[1], one, top);
+    a.w += cterm<OFF + 2, SHARED>(G, w[2], one, top) + cterm<OFF + 3, SHARED>(G, w[3], one, top);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -186,12 +210,23 @@ struct BF16State {
            make_uint2(mo[0] | (mo[1] << 16), mo[2] | (mo[3] << 16)));
     __stcs(reinterpret_cast<uint2 *>(static_cast<uint16_t *>(d.v) + off),
            make_uint2(vo[0] | (vo[1] << 16), vo[2] | (vo[3] << 16)));
-    a.p += digest_term<OFF>(G, po[0], s.one) + digest_term<OFF + 1>(G, po[1], s.one);
-    a.p += digest_term<OFF + 2>(G, po[2], s.one) + digest_term<OFF + 3>(G, po[3], s.one);
-    a.m += digest_term<OFF>(G, mo[0], s.one) + digest_term<OFF + 1>(G, mo[1], s.one);
-    a.m += digest_term<OFF + 2>(G, mo[2], s.one) + digest_term<OFF + 3>(G, mo[3], s.one);
-    a.v += digest_term<OFF>(G, vo[0], s.one) + digest_term<OFF + 1>(G, vo[1], s.one);
-    a.v += digest_term<OFF + 2>(G, vo[2], s.one) + digest_term<OFF + 3>(G, vo[3], s.one);
+    const uint32_t B = G + (0x9E3779B9u + OFF);  // the group's keys are G + OFF .. G + OFF + 3
+    if (top_bits_shared(B, 4)) {
+      fold<OFF, true>(G, po, mo, vo, s.one, B >> 30, a);
+    } else {
+      fold<OFF, false>(G, po, mo, vo, s.one, 0, a);
+    }
+  }
+
+  template <uint32_t OFF, bool SHARED>
+  __device__ static void fold(uint32_t G, const uint32_t (&p)[4], const uint32_t (&m)[4], const uint32_t (&v)[4],
+                              uint32_t one, uint32_t top, Acc &a) {
+    a.p += cterm<OFF, SHARED>(G, p[0], one, top) + cterm<OFF + 1, SHARED>(G, p[1], one, top);
+    a.p += cterm<OFF + 2, SHARED>(G, p[2], one, top) + cterm<OFF + 3, SHARED>(G, p[3], one, top);
+    a.m += cterm<OFF, SHARED>(G, m[0], one, top) + cterm<OFF + 1, SHARED>(G, m[1], one, top);
+    a.m += cterm<OFF + 2, SHARED>(G, m[2], one, top) + cterm<OFF + 3, SHARED>(G, m[3], one, top);
+    a.v += cterm<OFF, SHARED>(G, v[0], one, top) + cterm<OFF + 1, SHARED>(G, v[1], one, top);
+    a.v += cterm<OFF + 2, SHARED>(G, v[2], one, top) + cterm<OFF + 3, SHARED>(G, v[3], one, top);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {

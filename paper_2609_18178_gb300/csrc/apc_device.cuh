@@ -91,18 +91,43 @@ struct MulCompiler {
 // equal to 1 (so the assembler cannot turn it back into an ALU add) and the
 // offset K folded into the immediate: (G + K) + 0x9E3779B9 and
 // G + (0x9E3779B9 + K) are equal mod 2^32, and no add of K is issued.
-template <uint32_t K = 0, class Mul = MulWide>
-__device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits, uint32_t one) {
+//
+// The first xor-shift needs hi >> 30, the top two bits of the incremented
+// high word.  Callers that know them for a whole run of terms pass them as
+// `hi_top` (see digest_term's four-argument form); otherwise they are
+// computed here.
+template <uint32_t K, class Mul>
+__device__ __forceinline__ uint64_t digest_term_core(uint32_t gidx, uint32_t bits, uint32_t one, bool have_top,
+                                                     uint32_t hi_top) {
   uint32_t lo, hi;
   asm("add.cc.u32 %0, %2, 0x7F4A7C15;\n\t"
       "madc.lo.u32 %1, %4, %5, %3;"
       : "=r"(lo), "=r"(hi)
       : "r"(bits), "r"(gidx), "r"(one), "n"(0x9E3779B9u + K));
-  uint64_t z = ((uint64_t)hi << 32) | lo;
-  z = Mul::template mul<0x1CE4E5B9u, 0xBF58476Du>(z ^ (z >> 30));
+  const uint32_t l1 = lo ^ __funnelshift_r(lo, hi, 30);
+  const uint32_t h1 = hi ^ (have_top ? hi_top : hi >> 30);
+  uint64_t z = ((uint64_t)h1 << 32) | l1;
+  z = Mul::template mul<0x1CE4E5B9u, 0xBF58476Du>(z);
   z = Mul::template mul<0x133111EBu, 0x94D049BBu>(z ^ (z >> 27));
   return z ^ (z >> 31);
 }
+
+template <uint32_t K = 0, class Mul = MulWide>
+__device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits, uint32_t one) {
+  return digest_term_core<K, Mul>(gidx, bits, one, false, 0);
+}
+
+// The same term with hi >> 30 supplied: hi_top must equal the top two bits
+// of gidx + 0x9E3779B9 + K + carry.  For terms whose keys G + K lie in
+// [G0, G0 + R), every incremented high word lies in [B, B + R] with
+// B = G0 + 0x9E3779B9 (the carry adds at most 1); when B and B + R have the
+// same top two bits (top_bits_shared), those bits are B >> 30 for all of them.
+template <uint32_t K = 0, class Mul = MulWide>
+__device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits, uint32_t one, uint32_t hi_top) {
+  return digest_term_core<K, Mul>(gidx, bits, one, true, hi_top);
+}
+
+__device__ __forceinline__ bool top_bits_shared(uint32_t B, uint32_t R) { return ((B ^ (B + R)) >> 30) == 0; }
 
 // acc += z (mod 2^64), with the high half's carry-add on the FMA pipe.  Used
 // for single terms; pairs of terms are summed as acc += a + b, which the

@@ -894,3 +894,15 @@ def test_every_bf16_state_parameter_and_gradient_pair():
     pool.shutdown()
     del d
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("k", [0, 1, 2, 3])
+def test_groups_straddling_a_top_bits_boundary(k):
+    """The commit kernel shares hi >> 30 of the incremented key high word
+    (G + 0x9E3779B9 + carry) across a group of four elements unless the
+    group's range crosses a multiple of 2^30.  Tensors around each of the
+    four crossing points take both the shared and the exact path; outputs
+    and digests equal the oracle's."""
+    cross = ((k << 30) - 0x9E3779B9) & 0xFFFFFFFF      # the key index G at which the top bits change
+    tensors = [gen(n, cross - back + (1 << 32) * j, 2) for j, (n, back) in enumerate(((20_000, 9_999), (13, 7), (4_867, 4_800)))]
+    assert_same(*run_small(tensors, 2))
