@@ -30,6 +30,50 @@ __device__ __forceinline__ uint64_t term(uint32_t gidx, uint32_t bits, uint32_t 
   return digest_term<K, MulCompiler>(gidx, bits, one);
 }
 
+// The same with SHARED: the caller has checked that all of a thread's terms
+// in the tile share the top two bits of the incremented key high word
+// (top_bits_shared over the keys G0 .. G0 + (kDigestUnroll - 1) * kThreads *
+// kVec + 7) and passes them as `top`, so no term computes hi >> 30 itself.
+template <uint32_t K, bool SHARED>
+__device__ __forceinline__ uint64_t vterm(uint32_t gidx, uint32_t bits, uint32_t one, uint32_t top) {
+  if constexpr (SHARED) return digest_term<K, MulCompiler>(gidx, bits, one, top);
+  else return digest_term<K, MulCompiler>(gidx, bits, one);
+}
+
+// A thread's terms of one fp32 tile (kDigestUnroll vectors of 8 words).
+template <bool SHARED>
+__device__ __forceinline__ void fold32(const uint4 (&x)[kDigestUnroll][2], const bool (&ok)[kDigestUnroll], uint32_t G0,
+                                       uint32_t one, uint32_t top, uint64_t &t0, uint64_t &t1) {
+#pragma unroll
+  for (int u = 0; u < kDigestUnroll; ++u) {
+    if (!ok[u]) continue;
+    const uint32_t G = G0 + (uint32_t)(u * kThreads * kVec);
+    t0 += vterm<0, SHARED>(G, x[u][0].x, one, top) + vterm<1, SHARED>(G, x[u][0].y, one, top);
+    t1 += vterm<2, SHARED>(G, x[u][0].z, one, top) + vterm<3, SHARED>(G, x[u][0].w, one, top);
+    t0 += vterm<4, SHARED>(G, x[u][1].x, one, top) + vterm<5, SHARED>(G, x[u][1].y, one, top);
+    t1 += vterm<6, SHARED>(G, x[u][1].z, one, top) + vterm<7, SHARED>(G, x[u][1].w, one, top);
+  }
+}
+
+// A thread's terms of one bf16 tile (kDigestUnroll vectors of 8 words).
+template <bool SHARED>
+__device__ __forceinline__ void fold16(const uint4 (&x)[kDigestUnroll], const bool (&ok)[kDigestUnroll], uint32_t G0,
+                                       uint32_t one, uint32_t top, uint64_t &t0, uint64_t &t1) {
+#pragma unroll
+  for (int u = 0; u < kDigestUnroll; ++u) {
+    if (!ok[u]) continue;
+    const uint32_t G = G0 + (uint32_t)(u * kThreads * kVec);
+    t0 += vterm<0, SHARED>(G, x[u].x & 0xFFFFu, one, top) + vterm<1, SHARED>(G, x[u].x >> 16, one, top);
+    t1 += vterm<2, SHARED>(G, x[u].y & 0xFFFFu, one, top) + vterm<3, SHARED>(G, x[u].y >> 16, one, top);
+    t0 += vterm<4, SHARED>(G, x[u].z & 0xFFFFu, one, top) + vterm<5, SHARED>(G, x[u].z >> 16, one, top);
+    t1 += vterm<6, SHARED>(G, x[u].w & 0xFFFFu, one, top) + vterm<7, SHARED>(G, x[u].w >> 16, one, top);
+  }
+}
+
+// The keys of a thread's terms in a tile lie in [G0, G0 + kTileKeySpan - 1];
+// with the increment's carry their high words lie in [B, B + kTileKeySpan].
+constexpr uint32_t kTileKeySpan = (kDigestUnroll - 1) * kThreads * kVec + kVec;
+
 __device__ __forceinline__ void flush(uint64_t &acc, int slot, unsigned long long *s_acc) {
   uint64_t x = acc;
 #pragma unroll
@@ -78,15 +122,10 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
           x[u][1] = __ldcs(reinterpret_cast<const uint4 *>(d + i) + 1);
         }
       }
-#pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u) {
-        if (!ok[u]) continue;
-        const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        t0 += term<0>(G, x[u][0].x, one) + term<1>(G, x[u][0].y, one);
-        t1 += term<2>(G, x[u][0].z, one) + term<3>(G, x[u][0].w, one);
-        t0 += term<4>(G, x[u][1].x, one) + term<5>(G, x[u][1].y, one);
-        t1 += term<6>(G, x[u][1].z, one) + term<7>(G, x[u][1].w, one);
-      }
+      const uint32_t G0 = E.key_base + (uint32_t)(base + (uint64_t)threadIdx.x * kVec);
+      const uint32_t B = G0 + 0x9E3779B9u;
+      if (top_bits_shared(B, kTileKeySpan)) fold32<true>(x, ok, G0, one, B >> 30, t0, t1);
+      else fold32<false>(x, ok, G0, one, 0, t0, t1);
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
       uint4 x[kDigestUnroll];
@@ -97,15 +136,10 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
         ok[u] = i < vec_end;
         if (ok[u]) x[u] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
       }
-#pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u) {
-        if (!ok[u]) continue;
-        const uint32_t G = E.key_base + (uint32_t)(base + (uint64_t)(u * kThreads + threadIdx.x) * kVec);
-        t0 += term<0>(G, x[u].x & 0xFFFFu, one) + term<1>(G, x[u].x >> 16, one);
-        t1 += term<2>(G, x[u].y & 0xFFFFu, one) + term<3>(G, x[u].y >> 16, one);
-        t0 += term<4>(G, x[u].z & 0xFFFFu, one) + term<5>(G, x[u].z >> 16, one);
-        t1 += term<6>(G, x[u].w & 0xFFFFu, one) + term<7>(G, x[u].w >> 16, one);
-      }
+      const uint32_t G0 = E.key_base + (uint32_t)(base + (uint64_t)threadIdx.x * kVec);
+      const uint32_t B = G0 + 0x9E3779B9u;
+      if (top_bits_shared(B, kTileKeySpan)) fold16<true>(x, ok, G0, one, B >> 30, t0, t1);
+      else fold16<false>(x, ok, G0, one, 0, t0, t1);
     }
     if (local == 0) {
       const uint32_t t = threadIdx.x;

@@ -906,3 +906,27 @@ def test_groups_straddling_a_top_bits_boundary(k):
     cross = ((k << 30) - 0x9E3779B9) & 0xFFFFFFFF      # the key index G at which the top bits change
     tensors = [gen(n, cross - back + (1 << 32) * j, 2) for j, (n, back) in enumerate(((20_000, 9_999), (13, 7), (4_867, 4_800)))]
     assert_same(*run_small(tensors, 2))
+
+
+@pytest.mark.parametrize("k", [0, 1, 2, 3])
+def test_verify_tiles_straddling_a_top_bits_boundary(k):
+    """The verification pass shares hi >> 30 across a thread's terms in a
+    tile unless their keys' range crosses a multiple of 2^30 after the
+    increment; buffers around each crossing point (fp32 and bf16, aligned
+    and not) digest as the oracle does."""
+    rng = np.random.default_rng(40 + k)
+    cross = ((k << 30) - 0x9E3779B9) & 0xFFFFFFFF
+    bufs, want, keep = [], [0, 0], []
+    for back, n, shift in ((60_000, 120_001, 0), (7, 20, 1), (12_300, 30_000, 3)):
+        goff = cross - back + (1 << 33)
+        a = rng.integers(0, 2**32, size=n + shift, dtype=np.uint64).astype(np.uint32)
+        t = torch.from_numpy(a.view(np.int32)).cuda()
+        keep.append(t)
+        bufs.append(apc.BufferEntry(t[shift:], 0, goff, apc.F32))
+        want[0] = (want[0] + oracle.digest_f32(a[shift:], goff)) & M64
+        h = rng.integers(0, 2**16, size=n + shift, dtype=np.uint64).astype(np.uint16)
+        th = torch.from_numpy(h.view(np.int16)).cuda()
+        keep.append(th)
+        bufs.append(apc.BufferEntry(th[shift:], 1, goff, apc.BF16))
+        want[1] = (want[1] + oracle.digest_u16(h[shift:], goff)) & M64
+    assert apc.digests_to_host(apc.digest(bufs, 2)) == want
