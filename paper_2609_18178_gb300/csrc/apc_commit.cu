@@ -99,6 +99,14 @@ __device__ __forceinline__ uint64_t cterm(uint32_t G, uint32_t bits, uint32_t on
   else return digest_term<K>(G, bits, one);
 }
 
+// The term of a 16-bit word (w, and the bf16 layout's p', m', v'): with the
+// shared top bits, the 16-bit form digest_term_u16.
+template <uint32_t K, bool SHARED>
+__device__ __forceinline__ uint64_t hterm(uint32_t G, uint32_t bits, uint32_t one, uint32_t top) {
+  if constexpr (SHARED) return digest_term_u16<K>(G, bits, one, top);
+  else return digest_term<K>(G, bits, one);
+}
+
 // ------------------------------------------------------------ fp32 state
 
 struct F32State {
@@ -153,8 +161,8 @@ struct F32State {
     a.m += cterm<OFF + 2, SHARED>(G, m[2], one, top) + cterm<OFF + 3, SHARED>(G, m[3], one, top);
     a.v += cterm<OFF, SHARED>(G, v[0], one, top) + cterm<OFF + 1, SHARED>(G, v[1], one, top);
     a.v += cterm<OFF + 2, SHARED>(G, v[2], one, top) + cterm<OFF + 3, SHARED>(G, v[3], one, top);
-    a.w += cterm<OFF, SHARED>(G, w[0], one, top) + cterm<OFF + 1, SHARED>(G, w[1], one, top);
-    a.w += cterm<OFF + 2, SHARED>(G, w[2], one, top) + cterm<OFF + 3, SHARED>(G, w[3], one, top);
+    a.w += hterm<OFF, SHARED>(G, w[0], one, top) + hterm<OFF + 1, SHARED>(G, w[1], one, top);
+    a.w += hterm<OFF + 2, SHARED>(G, w[2], one, top) + hterm<OFF + 3, SHARED>(G, w[3], one, top);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {
@@ -221,12 +229,12 @@ struct BF16State {
   template <uint32_t OFF, bool SHARED>
   __device__ static void fold(uint32_t G, const uint32_t (&p)[4], const uint32_t (&m)[4], const uint32_t (&v)[4],
                               uint32_t one, uint32_t top, Acc &a) {
-    a.p += cterm<OFF, SHARED>(G, p[0], one, top) + cterm<OFF + 1, SHARED>(G, p[1], one, top);
-    a.p += cterm<OFF + 2, SHARED>(G, p[2], one, top) + cterm<OFF + 3, SHARED>(G, p[3], one, top);
-    a.m += cterm<OFF, SHARED>(G, m[0], one, top) + cterm<OFF + 1, SHARED>(G, m[1], one, top);
-    a.m += cterm<OFF + 2, SHARED>(G, m[2], one, top) + cterm<OFF + 3, SHARED>(G, m[3], one, top);
-    a.v += cterm<OFF, SHARED>(G, v[0], one, top) + cterm<OFF + 1, SHARED>(G, v[1], one, top);
-    a.v += cterm<OFF + 2, SHARED>(G, v[2], one, top) + cterm<OFF + 3, SHARED>(G, v[3], one, top);
+    a.p += hterm<OFF, SHARED>(G, p[0], one, top) + hterm<OFF + 1, SHARED>(G, p[1], one, top);
+    a.p += hterm<OFF + 2, SHARED>(G, p[2], one, top) + hterm<OFF + 3, SHARED>(G, p[3], one, top);
+    a.m += hterm<OFF, SHARED>(G, m[0], one, top) + hterm<OFF + 1, SHARED>(G, m[1], one, top);
+    a.m += hterm<OFF + 2, SHARED>(G, m[2], one, top) + hterm<OFF + 3, SHARED>(G, m[3], one, top);
+    a.v += hterm<OFF, SHARED>(G, v[0], one, top) + hterm<OFF + 1, SHARED>(G, v[1], one, top);
+    a.v += hterm<OFF + 2, SHARED>(G, v[2], one, top) + hterm<OFF + 3, SHARED>(G, v[3], one, top);
   }
 
   __device__ static void one(const CommitEntry &E, uint64_t i, const Scalars &s, Acc &a) {

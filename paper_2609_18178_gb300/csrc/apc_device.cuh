@@ -127,6 +127,27 @@ __device__ __forceinline__ uint64_t digest_term(uint32_t gidx, uint32_t bits, ui
   return digest_term_core<K, Mul>(gidx, bits, one, true, hi_top);
 }
 
+// splitmix64 term of a 16-bit word (bits < 2^16).  Its low key half plus
+// 0x7F4A7C15 never carries and always has top bits 01, so after the
+// increment lo = bits + 0x7F4A7C15, hi = gidx + 0x9E3779B9 + K, and the
+// first xor-shift's low word is lo ^ ((hi << 2) | 1) = lo ^ (4 * hi + 1).
+// All three are multiply-adds by `one` (the FMA pipe); `top` is hi >> 30,
+// shared by the caller (digest_term's hi_top rule).
+template <uint32_t K = 0, class Mul = MulWide>
+__device__ __forceinline__ uint64_t digest_term_u16(uint32_t gidx, uint32_t bits, uint32_t one, uint32_t top) {
+  uint32_t lo, hi, m4;
+  asm("mad.lo.u32 %0, %3, %4, 0x7F4A7C15;\n\t"
+      "mad.lo.u32 %1, %4, %6, %5;\n\t"
+      "mad.lo.u32 %2, %1, 4, %4;"
+      : "=r"(lo), "=r"(hi), "=r"(m4)
+      : "r"(bits), "r"(one), "r"(gidx), "n"(0x9E3779B9u + K));
+  const uint32_t l1 = lo ^ m4, h1 = hi ^ top;
+  uint64_t z = ((uint64_t)h1 << 32) | l1;
+  z = Mul::template mul<0x1CE4E5B9u, 0xBF58476Du>(z);
+  z = Mul::template mul<0x133111EBu, 0x94D049BBu>(z ^ (z >> 27));
+  return z ^ (z >> 31);
+}
+
 __device__ __forceinline__ bool top_bits_shared(uint32_t B, uint32_t R) { return ((B ^ (B + R)) >> 30) == 0; }
 
 // acc += z (mod 2^64), with the high half's carry-add on the FMA pipe.  Used

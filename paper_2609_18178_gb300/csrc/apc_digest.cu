@@ -55,6 +55,15 @@ __device__ __forceinline__ void fold32(const uint4 (&x)[kDigestUnroll][2], const
   }
 }
 
+// A bf16 word's term: with the shared top bits, the 16-bit form of
+// digest_term_u16 (its increment and first xor-shift take two ALU
+// instructions instead of four).
+template <uint32_t K, bool SHARED>
+__device__ __forceinline__ uint64_t hterm(uint32_t gidx, uint32_t bits, uint32_t one, uint32_t top) {
+  if constexpr (SHARED) return digest_term_u16<K, MulCompiler>(gidx, bits, one, top);
+  else return digest_term<K, MulCompiler>(gidx, bits, one);
+}
+
 // A thread's terms of one bf16 tile (kDigestUnroll vectors of 8 words).
 template <bool SHARED>
 __device__ __forceinline__ void fold16(const uint4 (&x)[kDigestUnroll], const bool (&ok)[kDigestUnroll], uint32_t G0,
@@ -63,10 +72,10 @@ __device__ __forceinline__ void fold16(const uint4 (&x)[kDigestUnroll], const bo
   for (int u = 0; u < kDigestUnroll; ++u) {
     if (!ok[u]) continue;
     const uint32_t G = G0 + (uint32_t)(u * kThreads * kVec);
-    t0 += vterm<0, SHARED>(G, x[u].x & 0xFFFFu, one, top) + vterm<1, SHARED>(G, x[u].x >> 16, one, top);
-    t1 += vterm<2, SHARED>(G, x[u].y & 0xFFFFu, one, top) + vterm<3, SHARED>(G, x[u].y >> 16, one, top);
-    t0 += vterm<4, SHARED>(G, x[u].z & 0xFFFFu, one, top) + vterm<5, SHARED>(G, x[u].z >> 16, one, top);
-    t1 += vterm<6, SHARED>(G, x[u].w & 0xFFFFu, one, top) + vterm<7, SHARED>(G, x[u].w >> 16, one, top);
+    t0 += hterm<0, SHARED>(G, x[u].x & 0xFFFFu, one, top) + hterm<1, SHARED>(G, x[u].x >> 16, one, top);
+    t1 += hterm<2, SHARED>(G, x[u].y & 0xFFFFu, one, top) + hterm<3, SHARED>(G, x[u].y >> 16, one, top);
+    t0 += hterm<4, SHARED>(G, x[u].z & 0xFFFFu, one, top) + hterm<5, SHARED>(G, x[u].z >> 16, one, top);
+    t1 += hterm<6, SHARED>(G, x[u].w & 0xFFFFu, one, top) + hterm<7, SHARED>(G, x[u].w >> 16, one, top);
   }
 }
 

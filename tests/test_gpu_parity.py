@@ -930,3 +930,20 @@ def test_verify_tiles_straddling_a_top_bits_boundary(k):
         bufs.append(apc.BufferEntry(th[shift:], 1, goff, apc.BF16))
         want[1] = (want[1] + oracle.digest_u16(h[shift:], goff)) & M64
     assert apc.digests_to_host(apc.digest(bufs, 2)) == want
+
+
+def test_every_bf16_word_digested_at_every_crossing():
+    """Every 16-bit word, digested by the verification pass (fp32 words are
+    covered by test_digest_of_every_low_word) at offsets that put the
+    shared-top-bits check on both sides of each 2^30 crossing, equals the
+    oracle's digest."""
+    words = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)
+    t = torch.from_numpy(words.view(np.int16)).cuda()
+    bufs, want = [], [0]
+    for k in range(4):
+        cross = ((k << 30) - 0x9E3779B9) & 0xFFFFFFFF
+        for j, back in enumerate((0, 1, 4_000, 60_000, 65_535)):
+            goff = cross - back + (j << 32)
+            bufs.append(apc.BufferEntry(t, 0, goff, apc.BF16))
+            want[0] = (want[0] + oracle.digest_u16(words, goff)) & M64
+    assert apc.digests_to_host(apc.digest(bufs, 1)) == want
