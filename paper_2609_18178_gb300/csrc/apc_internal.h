@@ -92,11 +92,11 @@ static_assert(sizeof(CommitPlan<kCommitLarge>) <= 32764, "kernel parameter limit
 #define APC_DIGEST_THREADS 384
 #endif
 #ifndef APC_DIGEST_UNROLL
-#define APC_DIGEST_UNROLL 4
+#define APC_DIGEST_UNROLL 3
 #endif
 constexpr int kThreads = APC_DIGEST_THREADS;     // threads per CTA of the digest kernel
 constexpr int kDigestUnroll = APC_DIGEST_UNROLL; // thread-vectors per thread per tile
-constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 12,288 elements
+constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 9,216 elements
 
 // One buffer of the digest kernel (32 bytes).
 //   head: scalar elements before the first 16-byte boundary (<= 7); then
