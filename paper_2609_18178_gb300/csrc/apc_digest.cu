@@ -2,13 +2,19 @@
 // after recovery): 4 (fp32) or 2 (bf16) bytes read per element and one
 // splitmix64 term per element, so the pass is bound by integer issue, not by
 // HBM.  It therefore streams straight into registers: each buffer's 16-byte
-// aligned body is cut into tiles of kDigestTile elements, a persistent grid
-// strides over the launch's tile space, every thread issues all of its
-// kDigestUnroll 16-byte (bf16) or 32-byte (fp32) loads of a tile before
-// folding any of them, and the scalar head and tail of a buffer go to the CTA
-// that owns its first tile.  (A bulk-copy pipeline like the commit kernel's
-// measured slower here: its per-tile synchronisation costs issue slots, the
-// one resource this pass is short of.)
+// aligned body is cut into tiles of kDigestTile elements, and each CTA of a
+// persistent grid takes one contiguous run of the launch's tile space (the
+// runs differ by at most one tile).  Inside its run a CTA finds the buffer of
+// its first tile once, then moves to the next buffer only when it crosses
+// one, carrying the element offset and key forward by a tile per step; this
+// costs measurably fewer integer instructions per tile than striding over the
+// tile space with a grid-wide step, which looks the buffer up and rebuilds
+// the offsets for every tile.  Every thread issues all of its kDigestUnroll
+// 16-byte (bf16) or 32-byte (fp32) loads of a tile before folding any of
+// them, and the scalar head and tail of a buffer go to the CTA that owns its
+// first tile.  (A bulk-copy pipeline like the commit kernel's measured slower
+// here: its per-tile synchronisation costs issue slots, the one resource this
+// pass is short of.)
 //
 // A thread keeps one running 64-bit sum for the slot of the buffer it is in;
 // all threads of a CTA visit the same tiles, so slot changes are CTA-uniform
@@ -103,54 +109,65 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
   if (threadIdx.x < APC_MAX_SLOTS) s_acc[threadIdx.x] = 0;
   __syncthreads();
   const uint32_t one = plan.one;
-  uint32_t cur = 0;
   int slot = -1;
   uint64_t acc = 0;
-  for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
-    while (cur + 1 < plan.count && tile >= plan.e[cur + 1].tile_begin) ++cur;
+  // this CTA's contiguous run of the launch's tiles: [tile, t_end)
+  const uint64_t per = plan.total_tiles / gridDim.x, rem = plan.total_tiles % gridDim.x;
+  uint64_t tile = blockIdx.x * per + (blockIdx.x < rem ? blockIdx.x : rem);
+  const uint64_t t_end = tile + per + (blockIdx.x < rem ? 1 : 0);
+  uint32_t cur = 0;
+  while (cur + 1 < plan.count && tile >= plan.e[cur + 1].tile_begin) ++cur;
+  const uint64_t t8 = (uint64_t)threadIdx.x * kVec;
+  for (; tile < t_end; ++cur) {
     const DigestEntry &E = plan.e[cur];
+    const uint64_t stop_e = cur + 1 < plan.count ? plan.e[cur + 1].tile_begin : plan.total_tiles;
+    const uint64_t stop = stop_e < t_end ? stop_e : t_end;
+    if (tile >= stop) continue;
     if ((int)E.slot != slot) {
       flush(acc, slot, s_acc);
       slot = E.slot;
     }
-    const uint64_t local = tile - E.tile_begin;
     const uint64_t head = E.head;
     const uint64_t vec_end = head + ((E.n - head) & ~(uint64_t)(kVec - 1));
-    const uint64_t base = head + local * kDigestTile;
+    uint64_t base = head + (tile - E.tile_begin) * kDigestTile + t8;   // this thread's first element
+    uint32_t G0 = E.key_base + (uint32_t)base;
+    const bool first = tile == E.tile_begin;
     uint64_t t0 = 0, t1 = 0;
     if (E.dtype == 0) {
       const uint32_t *d = reinterpret_cast<const uint32_t *>(E.data);
-      uint4 x[kDigestUnroll][2];
-      bool ok[kDigestUnroll];
+      for (; tile < stop; ++tile, base += kDigestTile, G0 += (uint32_t)kDigestTile) {
+        uint4 x[kDigestUnroll][2];
+        bool ok[kDigestUnroll];
 #pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u) {
-        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
-        ok[u] = i < vec_end;
-        if (ok[u]) {
-          x[u][0] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
-          x[u][1] = __ldcs(reinterpret_cast<const uint4 *>(d + i) + 1);
+        for (int u = 0; u < kDigestUnroll; ++u) {
+          const uint64_t i = base + (uint64_t)(u * kThreads) * kVec;
+          ok[u] = i < vec_end;
+          if (ok[u]) {
+            x[u][0] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
+            x[u][1] = __ldcs(reinterpret_cast<const uint4 *>(d + i) + 1);
+          }
         }
+        const uint32_t B = G0 + 0x9E3779B9u;
+        if (top_bits_shared(B, kTileKeySpan)) fold32<true>(x, ok, G0, one, B >> 30, t0, t1);
+        else fold32<false>(x, ok, G0, one, 0, t0, t1);
       }
-      const uint32_t G0 = E.key_base + (uint32_t)(base + (uint64_t)threadIdx.x * kVec);
-      const uint32_t B = G0 + 0x9E3779B9u;
-      if (top_bits_shared(B, kTileKeySpan)) fold32<true>(x, ok, G0, one, B >> 30, t0, t1);
-      else fold32<false>(x, ok, G0, one, 0, t0, t1);
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
-      uint4 x[kDigestUnroll];
-      bool ok[kDigestUnroll];
+      for (; tile < stop; ++tile, base += kDigestTile, G0 += (uint32_t)kDigestTile) {
+        uint4 x[kDigestUnroll];
+        bool ok[kDigestUnroll];
 #pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u) {
-        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
-        ok[u] = i < vec_end;
-        if (ok[u]) x[u] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
+        for (int u = 0; u < kDigestUnroll; ++u) {
+          const uint64_t i = base + (uint64_t)(u * kThreads) * kVec;
+          ok[u] = i < vec_end;
+          if (ok[u]) x[u] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
+        }
+        const uint32_t B = G0 + 0x9E3779B9u;
+        if (top_bits_shared(B, kTileKeySpan)) fold16<true>(x, ok, G0, one, B >> 30, t0, t1);
+        else fold16<false>(x, ok, G0, one, 0, t0, t1);
       }
-      const uint32_t G0 = E.key_base + (uint32_t)(base + (uint64_t)threadIdx.x * kVec);
-      const uint32_t B = G0 + 0x9E3779B9u;
-      if (top_bits_shared(B, kTileKeySpan)) fold16<true>(x, ok, G0, one, B >> 30, t0, t1);
-      else fold16<false>(x, ok, G0, one, 0, t0, t1);
     }
-    if (local == 0) {
+    if (first) {   // the CTA that owns an entry's first tile also does its scalar head and tail
       const uint32_t t = threadIdx.x;
       if (t < head) { acc_add(t0, term<0>(E.key_base + t, word_at(E, t), one), one); }
       if (t >= 32 && t - 32 < E.n - vec_end) {
