@@ -9,10 +9,11 @@
 // one, carrying the element offset and key forward by a tile per step; this
 // costs measurably fewer integer instructions per tile than striding over the
 // tile space with a grid-wide step, which looks the buffer up and rebuilds
-// the offsets for every tile.  Every thread issues all of its kDigestUnroll
-// 16-byte (bf16) or 32-byte (fp32) loads of a tile before folding any of
-// them, and the scalar head and tail of a buffer go to the CTA that owns its
-// first tile.  (A bulk-copy pipeline like the commit kernel's measured slower
+// the offsets for every tile.  All tiles of a buffer but its last are full
+// and run without per-vector bounds checks.  Every thread issues all of its
+// kDigestUnroll 16-byte (bf16) or 32-byte (fp32) loads of a tile before
+// folding any of them, and the scalar head and tail of a buffer go to the CTA
+// that owns its first tile.  (A bulk-copy pipeline like the commit kernel's measured slower
 // here: its per-tile synchronisation costs issue slots, the one resource this
 // pass is short of.)
 //
@@ -89,6 +90,42 @@ __device__ __forceinline__ void fold16(const uint4 (&x)[kDigestUnroll], const bo
 // with the increment's carry their high words lie in [B, B + kTileKeySpan].
 constexpr uint32_t kTileKeySpan = (kDigestUnroll - 1) * kThreads * kVec + kVec;
 
+// One tile of a thread's words: kDigestUnroll vectors of 8, the first at q
+// (element `base` of the buffer), the others kThreads vectors apart.  Only
+// the vectors with ok[u] are loaded and folded.
+__device__ __forceinline__ void tile32(const uint4 *q, const bool (&ok)[kDigestUnroll], uint32_t G0, uint32_t one,
+                                       uint64_t &t0, uint64_t &t1) {
+  uint4 x[kDigestUnroll][2];
+#pragma unroll
+  for (int u = 0; u < kDigestUnroll; ++u) {
+    if (ok[u]) {
+      x[u][0] = __ldcs(q + 2 * u * kThreads);
+      x[u][1] = __ldcs(q + 2 * u * kThreads + 1);
+    }
+  }
+  const uint32_t B = G0 + 0x9E3779B9u;
+  if (top_bits_shared(B, kTileKeySpan)) fold32<true>(x, ok, G0, one, B >> 30, t0, t1);
+  else fold32<false>(x, ok, G0, one, 0, t0, t1);
+}
+
+__device__ __forceinline__ void tile16(const uint4 *q, const bool (&ok)[kDigestUnroll], uint32_t G0, uint32_t one,
+                                       uint64_t &t0, uint64_t &t1) {
+  uint4 x[kDigestUnroll];
+#pragma unroll
+  for (int u = 0; u < kDigestUnroll; ++u) {
+    if (ok[u]) x[u] = __ldcs(q + u * kThreads);
+  }
+  const uint32_t B = G0 + 0x9E3779B9u;
+  if (top_bits_shared(B, kTileKeySpan)) fold16<true>(x, ok, G0, one, B >> 30, t0, t1);
+  else fold16<false>(x, ok, G0, one, 0, t0, t1);
+}
+
+// Which of a thread's vectors in an entry's last tile lie in its body.
+__device__ __forceinline__ void last_tile_ok(uint64_t base, uint64_t vec_end, bool (&ok)[kDigestUnroll]) {
+#pragma unroll
+  for (int u = 0; u < kDigestUnroll; ++u) ok[u] = base + (uint64_t)(u * kThreads) * kVec < vec_end;
+}
+
 __device__ __forceinline__ void flush(uint64_t &acc, int slot, unsigned long long *s_acc) {
   uint64_t x = acc;
 #pragma unroll
@@ -102,8 +139,11 @@ __device__ __forceinline__ uint32_t word_at(const DigestEntry &E, uint64_t i) {
                       : (uint32_t) reinterpret_cast<const uint16_t *>(E.data)[i];
 }
 
+// Two CTAs per SM (24 warps).  The bound lets the compiler use 80 registers:
+// without per-vector checks a full tile's 24 terms form one block that it
+// schedules for more overlap than 64 registers hold.
 template <int MAXE>
-__global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
+__global__ void __launch_bounds__(kThreads, 2) digest_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
                                                           unsigned long long *out) {
   __shared__ unsigned long long s_acc[APC_MAX_SLOTS];
   if (threadIdx.x < APC_MAX_SLOTS) s_acc[threadIdx.x] = 0;
@@ -133,38 +173,31 @@ __global__ void __launch_bounds__(kThreads) digest_kernel(const __grid_constant_
     uint32_t G0 = E.key_base + (uint32_t)base;
     const bool first = tile == E.tile_begin;
     uint64_t t0 = 0, t1 = 0;
+    // Every tile of an entry but its last is full (all vectors of all threads
+    // lie in the body) and runs without per-vector checks.
+    const uint64_t full_end = stop_e - 1 < stop ? stop_e - 1 : stop;
+    bool all[kDigestUnroll], ok[kDigestUnroll];
+#pragma unroll
+    for (int u = 0; u < kDigestUnroll; ++u) all[u] = true;
     if (E.dtype == 0) {
       const uint32_t *d = reinterpret_cast<const uint32_t *>(E.data);
-      for (; tile < stop; ++tile, base += kDigestTile, G0 += (uint32_t)kDigestTile) {
-        uint4 x[kDigestUnroll][2];
-        bool ok[kDigestUnroll];
-#pragma unroll
-        for (int u = 0; u < kDigestUnroll; ++u) {
-          const uint64_t i = base + (uint64_t)(u * kThreads) * kVec;
-          ok[u] = i < vec_end;
-          if (ok[u]) {
-            x[u][0] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
-            x[u][1] = __ldcs(reinterpret_cast<const uint4 *>(d + i) + 1);
-          }
-        }
-        const uint32_t B = G0 + 0x9E3779B9u;
-        if (top_bits_shared(B, kTileKeySpan)) fold32<true>(x, ok, G0, one, B >> 30, t0, t1);
-        else fold32<false>(x, ok, G0, one, 0, t0, t1);
+      const uint4 *q = reinterpret_cast<const uint4 *>(d + base);
+      for (; tile < full_end; ++tile, q += kDigestTile / 4, G0 += (uint32_t)kDigestTile)
+        tile32(q, all, G0, one, t0, t1);
+      if (tile < stop) {  // the entry's last tile
+        last_tile_ok((uint64_t)(reinterpret_cast<const uint32_t *>(q) - d), vec_end, ok);
+        tile32(q, ok, G0, one, t0, t1);
+        ++tile;
       }
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
-      for (; tile < stop; ++tile, base += kDigestTile, G0 += (uint32_t)kDigestTile) {
-        uint4 x[kDigestUnroll];
-        bool ok[kDigestUnroll];
-#pragma unroll
-        for (int u = 0; u < kDigestUnroll; ++u) {
-          const uint64_t i = base + (uint64_t)(u * kThreads) * kVec;
-          ok[u] = i < vec_end;
-          if (ok[u]) x[u] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
-        }
-        const uint32_t B = G0 + 0x9E3779B9u;
-        if (top_bits_shared(B, kTileKeySpan)) fold16<true>(x, ok, G0, one, B >> 30, t0, t1);
-        else fold16<false>(x, ok, G0, one, 0, t0, t1);
+      const uint4 *q = reinterpret_cast<const uint4 *>(d + base);
+      for (; tile < full_end; ++tile, q += kDigestTile / 8, G0 += (uint32_t)kDigestTile)
+        tile16(q, all, G0, one, t0, t1);
+      if (tile < stop) {  // the entry's last tile
+        last_tile_ok((uint64_t)(reinterpret_cast<const uint16_t *>(q) - d), vec_end, ok);
+        tile16(q, ok, G0, one, t0, t1);
+        ++tile;
       }
     }
     if (first) {   // the CTA that owns an entry's first tile also does its scalar head and tail
