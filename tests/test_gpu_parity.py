@@ -93,7 +93,12 @@ def test_c1_chained_three_steps():
         assert apc.digests_to_host(ver) == dref
 
 
-@pytest.mark.parametrize("n", list(range(1, 65)) + [127, 129, 4095, 4096, 4097, 8191, 8199, 100003])
+# Elements per tile of the commit kernel (19 consumer warps x 32 threads x 2 groups of 4).
+COMMIT_TILE = 4864
+
+
+@pytest.mark.parametrize("n", list(range(1, 65)) + [127, 129, 4095, 4096, 4097, 8191, 8199, 100003] +
+                         [k * COMMIT_TILE + d for k in (1, 2) for d in (-8, -1, 0, 1, 8)])
 def test_small_sizes(n):
     goff = (1 << 32) - n // 2 - 3
     assert_same(*run_small([gen(n, goff, 2)], 2))
@@ -247,6 +252,49 @@ def test_digest_of_arbitrary_buffers():
         bufs.append(apc.BufferEntry(t[shift:], slot, goff, apc.F32 if f32 else apc.BF16))
     out = apc.digest(bufs, 8)
     assert apc.digests_to_host(out) == want
+
+
+# Elements per tile of the verification kernel (384 threads x 3 vectors of 8):
+# every tile of a buffer but its last runs without bounds checks.
+DIGEST_TILE = 9216
+
+
+@pytest.mark.parametrize("limit", [None, 1, 5])
+def test_digest_buffers_at_tile_boundaries(monkeypatch, limit):
+    """Buffers whose vector bodies end exactly on, just before and just after
+    a tile boundary, with and without a scalar head, on the default grid and
+    on grids of 1 and 5 CTAs (whose contiguous tile runs then start and end
+    inside buffers): every slot's digest equals the oracle's."""
+    if limit is None:
+        monkeypatch.delenv("APC_GRID_LIMIT", raising=False)
+    else:
+        monkeypatch.setenv("APC_GRID_LIMIT", str(limit))
+    rng = np.random.default_rng(33)
+    bufs, each, keep = [], [], []
+    sizes = [k * DIGEST_TILE + d for k in (1, 2, 3) for d in (-8, -1, 0, 1, 7, 8, 9)] + [5 * DIGEST_TILE + 8 * 384]
+    for i, n in enumerate(sizes):
+        for f32 in (True, False):
+            shift = int(rng.integers(1, 8)) if i % 2 else 0   # a nonzero shift gives a scalar head
+            goff = int(rng.integers(0, 1 << 33))
+            slot = (2 * i + f32) % 4
+            if f32:
+                a = rng.integers(0, 2**32, size=n + shift, dtype=np.uint64).astype(np.uint32)
+                t = torch.from_numpy(a.view(np.int32)).cuda()
+                each.append((slot, oracle.digest_f32(a[shift:], goff)))
+            else:
+                a = rng.integers(0, 2**16, size=n + shift, dtype=np.uint64).astype(np.uint16)
+                t = torch.from_numpy(a.view(np.int16)).cuda()
+                each.append((slot, oracle.digest_u16(a[shift:], goff)))
+            keep.append(t)
+            bufs.append(apc.BufferEntry(t[shift:], slot, goff, apc.F32 if f32 else apc.BF16))
+    want = [0] * 4
+    for slot, d in each:
+        want[slot] = (want[slot] + d) & M64
+    assert apc.digests_to_host(apc.digest(bufs, 4)) == want
+    # each buffer alone, so that no wrong term hides behind another buffer's in the same slot
+    for b, (slot, d) in zip(bufs, each):
+        alone = apc.BufferEntry(b.data, 0, b.global_offset, b.dtype)
+        assert apc.digests_to_host(apc.digest([alone], 1))[0] == d, (b.data.numel(), b.dtype)
 
 
 def test_invalid_arguments_are_rejected():
