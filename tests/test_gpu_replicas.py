@@ -1,4 +1,4 @@
-"""Replica verification on the GPU (survey next row f4): replica processes
+"""Replica verification on the GPU: replica processes
 of one hybrid-sharding replication group commit identical shards, verify,
 and agree over the Gloo control plane; a bit flipped in one replica's HBM
 state through a host-side copy is then seen by every replica."""
