@@ -12,8 +12,9 @@
 // with +0 once its copy has landed: 2 more bytes per element.
 //
 // Warp-specialized pipeline (one persistent CTA per SM by default):
-//  * The producer warp walks the launch's tiles (kCommitTile = 4864 elements
-//    of one entry's 16-byte aligned body) and, for each, waits until a ring
+//  * The producer warp walks the launch's tiles (L::kTile elements of one
+//    entry's 16-byte aligned body: 4,864 for fp32 state, 9,728 for bf16
+//    state) and, for each, waits until a ring
 //    stage is free and issues four bulk asynchronous copies -- p, m, v and g
 //    -- that complete on the stage's "full" mbarrier.  Loads never occupy
 //    consumer registers, and up to kCommitStages tiles per CTA are in flight.
@@ -123,6 +124,8 @@ __device__ __forceinline__ uint64_t hterm(uint32_t G, uint32_t bits, uint32_t on
 struct F32State {
   static constexpr uint32_t kES = 4;        // bytes per state element
   static constexpr int kDigests = 4;
+  static constexpr int kGroups = kCommitGroups;
+  static constexpr uint64_t kTile = kCommitTile;
   struct Regs {
     float4 p, m, v;
     uint2 g;
@@ -130,9 +133,9 @@ struct F32State {
 
   __device__ static void load(const uint8_t *st, uint32_t e, Regs &r) {
     r.p = *reinterpret_cast<const float4 *>(st + 4 * e);
-    r.m = *reinterpret_cast<const float4 *>(st + 4 * (kCommitTile + e));
-    r.v = *reinterpret_cast<const float4 *>(st + 4 * (2 * kCommitTile + e));
-    r.g = *reinterpret_cast<const uint2 *>(st + 12 * kCommitTile + 2 * e);
+    r.m = *reinterpret_cast<const float4 *>(st + 4 * (kTile + e));
+    r.v = *reinterpret_cast<const float4 *>(st + 4 * (2 * kTile + e));
+    r.g = *reinterpret_cast<const uint2 *>(st + 12 * kTile + 2 * e);
   }
 
   // Four consecutive elements at the compile-time element offset OFF from
@@ -197,15 +200,17 @@ struct F32State {
 struct BF16State {
   static constexpr uint32_t kES = 2;
   static constexpr int kDigests = 3;
+  static constexpr int kGroups = kCommitGroupsBF16;
+  static constexpr uint64_t kTile = kCommitTileBF16;
   struct Regs {
     uint2 p, m, v, g;
   };
 
   __device__ static void load(const uint8_t *st, uint32_t e, Regs &r) {
     r.p = *reinterpret_cast<const uint2 *>(st + 2 * e);
-    r.m = *reinterpret_cast<const uint2 *>(st + 2 * (kCommitTile + e));
-    r.v = *reinterpret_cast<const uint2 *>(st + 2 * (2 * kCommitTile + e));
-    r.g = *reinterpret_cast<const uint2 *>(st + 6 * kCommitTile + 2 * e);
+    r.m = *reinterpret_cast<const uint2 *>(st + 2 * (kTile + e));
+    r.v = *reinterpret_cast<const uint2 *>(st + 2 * (2 * kTile + e));
+    r.g = *reinterpret_cast<const uint2 *>(st + 6 * kTile + 2 * e);
   }
 
   template <uint32_t OFF>
@@ -278,12 +283,12 @@ __device__ __forceinline__ void store_groups(const Dst &d, uint32_t G1, const ty
     if (ZERO) __stcs(reinterpret_cast<uint2 *>(d.g + off), make_uint2(0u, 0u));
     L::template compute_store<off>(d, G1, r[K], s, a);
   }
-  if constexpr (K + 1 < kCommitGroups) store_groups<L, ZERO, K + 1>(d, G1, r, ok, s, a);
+  if constexpr (K + 1 < L::kGroups) store_groups<L, ZERO, K + 1>(d, G1, r, ok, s, a);
 }
 
 template <class L>
 __host__ __device__ constexpr uint32_t stage_bytes() {
-  return (uint32_t)kCommitTile * (3 * L::kES + 2);
+  return (uint32_t)L::kTile * (3 * L::kES + 2);
 }
 
 template <class L>
@@ -291,7 +296,7 @@ __host__ __device__ constexpr uint32_t smem_bytes() {
   return (uint32_t)kCommitStages * stage_bytes<L>();
 }
 
-static_assert(smem_bytes<F32State>() <= 227 * 1024, "shared memory per CTA");
+static_assert(smem_bytes<F32State>() <= 227 * 1024 && smem_bytes<BF16State>() <= 227 * 1024, "shared memory per CTA");
 
 template <int MAXE>
 __device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint32_t cur, uint64_t tile) {
@@ -332,9 +337,9 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
         if (*(volatile int *)&abort_flag) break;
         cur = find_tile(plan, cur, tile);
         const CommitEntry &E = plan.e[cur];
-        const uint64_t start = E.head + (tile - E.tile_begin) * kCommitTile;
+        const uint64_t start = E.head + (tile - E.tile_begin) * L::kTile;
         const uint64_t vec_end = E.head + ((E.n - E.head) & ~(uint64_t)7);
-        const uint32_t cnt = (uint32_t)umin64(kCommitTile, vec_end - start);
+        const uint32_t cnt = (uint32_t)umin64(L::kTile, vec_end - start);
         if (!mbar_wait(&empty[stage], phase ^ 1)) {
           fail_wait(&abort_flag);
           break;
@@ -349,11 +354,11 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
                                 E.key_base + (uint32_t)start};
         mbar_arrive_expect_tx(&full[stage], cnt * (3 * L::kES + 2));
         bulk_g2s(st, static_cast<const uint8_t *>(E.p) + start * L::kES, cnt * L::kES, &full[stage], policy);
-        bulk_g2s(st + L::kES * kCommitTile, static_cast<const uint8_t *>(E.m) + start * L::kES, cnt * L::kES,
+        bulk_g2s(st + L::kES * L::kTile, static_cast<const uint8_t *>(E.m) + start * L::kES, cnt * L::kES,
                  &full[stage], policy);
-        bulk_g2s(st + 2 * L::kES * kCommitTile, static_cast<const uint8_t *>(E.v) + start * L::kES,
+        bulk_g2s(st + 2 * L::kES * L::kTile, static_cast<const uint8_t *>(E.v) + start * L::kES,
                  cnt * L::kES, &full[stage], policy);
-        bulk_g2s(st + 3 * L::kES * kCommitTile, E.g + start, cnt * 2, &full[stage], policy);
+        bulk_g2s(st + 3 * L::kES * L::kTile, E.g + start, cnt * 2, &full[stage], policy);
         ++issued;
         if (++stage == kCommitStages) {
           stage = 0;
@@ -386,10 +391,10 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
       if (*(volatile int *)&abort_flag) break;
       const StageDesc sd = desc[stage];
       const uint8_t *st = smem + (size_t)stage * stage_bytes<L>();
-      typename L::Regs r[kCommitGroups];
-      bool ok[kCommitGroups];
+      typename L::Regs r[L::kGroups];
+      bool ok[L::kGroups];
 #pragma unroll
-      for (int k = 0; k < kCommitGroups; ++k) {
+      for (int k = 0; k < L::kGroups; ++k) {
         const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
         ok[k] = e < sd.cnt;
         if (ok[k]) L::load(st, e, r[k]);

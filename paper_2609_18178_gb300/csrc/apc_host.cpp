@@ -274,7 +274,7 @@ apc_status commit_common(int layout, const std::vector<TableRow> &rows, const ap
       const uint64_t head = std::min<uint64_t>(h0, t.n);
       const uint64_t body = (t.n - head) / apc::kVec * apc::kVec;
       e.head = (uint32_t)head;
-      e.tile_begin = ceil_div(body, apc::kCommitTile);  // tile count until placed
+      e.tile_begin = ceil_div(body, apc::commit_tile(layout));  // tile count until placed
       e.scalar_begin = t.n - body;                       // head + tail items
     } else {
       e.head = apc::kScalarMode;

@@ -29,6 +29,9 @@ constexpr uint32_t kScalarMode = 0xFFFFFFFFu;  // `head` value of an entry run w
 #ifndef APC_COMMIT_GROUPS
 #define APC_COMMIT_GROUPS 2
 #endif
+#ifndef APC_COMMIT_GROUPS_BF16
+#define APC_COMMIT_GROUPS_BF16 4
+#endif
 #ifndef APC_COMMIT_STAGES
 #define APC_COMMIT_STAGES 2
 #endif
@@ -38,23 +41,31 @@ constexpr uint32_t kScalarMode = 0xFFFFFFFFu;  // `head` value of an entry run w
 constexpr int kCommitConsumerWarps = APC_COMMIT_CONSUMER_WARPS;
 constexpr int kCommitConsumers = kCommitConsumerWarps * 32;
 constexpr int kCommitThreads = kCommitConsumers + 32;                   // + the producer warp
-constexpr int kCommitGroups = APC_COMMIT_GROUPS;                        // 4-element groups per thread per tile
-constexpr uint64_t kCommitTile = (uint64_t)kCommitConsumers * 4 * kCommitGroups;
+// 4-element groups per consumer thread per tile, for each state layout.  The
+// bf16 layout, with half the staged bytes per element, takes 4 (1.8% faster
+// than 2 there; 3 gave 1.2%, 5 was slower); the fp32 layout keeps 2 (3 ran
+// 6% slower).
+constexpr int kCommitGroups = APC_COMMIT_GROUPS;
+constexpr int kCommitGroupsBF16 = APC_COMMIT_GROUPS_BF16;
+constexpr uint64_t kCommitTile = (uint64_t)kCommitConsumers * 4 * kCommitGroups;          // 4,864 elements
+constexpr uint64_t kCommitTileBF16 = (uint64_t)kCommitConsumers * 4 * kCommitGroupsBF16;  // 9,728 elements
 constexpr int kCommitStages = APC_COMMIT_STAGES;
 constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
 // A stage holds one tile of p, m, v and g: 14 bytes per element for fp32
-// state (133 KB per CTA at the defaults), 8 for bf16 state.
+// state (133 KB per CTA at the defaults), 8 for bf16 state (152 KB).
 
 // State layouts of the commit kernel.
 constexpr int kLayoutF32 = 0;   // fp32 p, m, v; bf16 g; bf16 copy w
 constexpr int kLayoutBF16 = 1;  // bf16 p, m, v; bf16 g; no copy
+
+constexpr uint64_t commit_tile(int layout) { return layout == kLayoutBF16 ? kCommitTileBF16 : kCommitTile; }
 
 // One chunk-table entry of the commit kernel (72 bytes).
 //   p, m, v: fp32 or bf16 state (by the launch's layout); w: the bf16 copy
 //         (fp32 layout only).
 //   head: elements [0, head) are scalar items, then 16-byte aligned vectors
 //         up to vec_end = head + 8 * floor((n - head) / 8) in tiles of
-//         kCommitTile, then scalar items up to n; kScalarMode when the
+//         commit_tile(layout), then scalar items up to n; kScalarMode when the
 //         buffers are not mutually 16-byte aligned (all n elements scalar).
 //   tile_begin: the entry's first tile in the launch's tile space.
 //   scalar_begin: the entry's first item in the launch's scalar-item space.

@@ -588,7 +588,12 @@ def run_bf16(tensors, step, hp=HP, zero_grad=False, shift=0):
     assert apc.digests_to_host(out) == want
 
 
-@pytest.mark.parametrize("n", [1, 3, 7, 8, 9, 63, 4864, 4871, 9728 + 5, 100003])
+# Elements per tile of the commit kernel's bf16-state layout (19 x 32 threads x 4 groups of 4).
+COMMIT_TILE_BF16 = 9728
+
+
+@pytest.mark.parametrize("n", [1, 3, 7, 8, 9, 63, 4864, 4871, 9728 + 5, 100003] +
+                         [k * COMMIT_TILE_BF16 + d for k in (1, 2) for d in (-8, -1, 0, 1, 8)])
 def test_bf16_state_sizes(n):
     run_bf16([gen16(n, (1 << 32) - n // 3, 2)], 2)
 
