@@ -1,27 +1,35 @@
 // The read-only state digest over a list of buffers (the verification pass
 // after recovery): 4 (fp32) or 2 (bf16) bytes read per element and one
 // splitmix64 term per element, so the pass is bound by integer issue, not by
-// HBM.  It therefore streams straight into registers: each buffer's 16-byte
-// aligned body is cut into tiles of kDigestTile elements, and each CTA of a
-// persistent grid takes one contiguous run of the launch's tile space (the
-// runs differ by at most one tile).  Inside its run a CTA finds the buffer of
-// its first tile once, then moves to the next buffer only when it crosses
-// one, carrying the element offset and key forward by a tile per step; this
-// costs measurably fewer integer instructions per tile than striding over the
-// tile space with a grid-wide step, which looks the buffer up and rebuilds
-// the offsets for every tile.  All tiles of a buffer but its last are full
-// and run without per-vector bounds checks.  Every thread issues all of its
-// kDigestUnroll 16-byte (bf16) or 32-byte (fp32) loads of a tile before
-// folding any of them, and the scalar head and tail of a buffer go to the CTA
-// that owns its first tile.  (A bulk-copy pipeline like the commit kernel's measured slower
-// here: its per-tile synchronisation costs issue slots, the one resource this
-// pass is short of.)
+// HBM.
+//
+// Work split: each buffer's 16-byte aligned body is cut into tiles of
+// kDigestTile elements, and each CTA of a persistent grid takes one
+// contiguous run of the launch's tile space (the runs differ by at most one
+// tile).  Inside its run a CTA finds the buffer of its first tile once, then
+// moves to the next buffer only when it crosses one, carrying the element
+// offset and key forward by a tile per step; this costs measurably fewer
+// integer instructions per tile than striding over the tile space with a
+// grid-wide step, which looks the buffer up and rebuilds the offsets for
+// every tile.
+//
+// Loads: a thread's part of a tile is kDigestUnroll vectors of 8 words.  All
+// tiles of a buffer but its last are full; they run without per-vector bounds
+// checks, and each thread keeps its next full tile in flight with cp.async
+// into shared-memory slots that only it reads (two stages, no barrier), then
+// folds the current one from there.  A buffer's last tile is loaded straight
+// into registers with per-vector checks, and its scalar head and tail go to
+// the CTA that owns its first tile.  (A CTA-wide bulk-copy pipeline like the
+// commit kernel's measured slower here: its per-tile synchronisation costs
+// issue slots, the one resource this pass is short of.)
 //
 // A thread keeps one running 64-bit sum for the slot of the buffer it is in;
 // all threads of a CTA visit the same tiles, so slot changes are CTA-uniform
 // and the running sum is flushed (warp shuffle reduce, then a shared-memory
 // atomic) only when the CTA moves to a buffer of another slot and at exit.
 #include <cuda_runtime.h>
+
+#include <atomic>
 
 #include "../../include/apc.h"
 #include "apc_device.cuh"
@@ -126,6 +134,21 @@ __device__ __forceinline__ void last_tile_ok(uint64_t base, uint64_t vec_end, bo
   for (int u = 0; u < kDigestUnroll; ++u) ok[u] = base + (uint64_t)(u * kThreads) * kVec < vec_end;
 }
 
+// Per-thread double buffering of full tiles in shared memory: while a thread
+// folds one tile it has the next one in flight with cp.async, into slots that
+// only it reads, so no barrier is needed; cp.async.wait_group orders each
+// thread's own copies.  Slot k of stage b of thread t is
+// stg[(b * kStageSlots + k) * kThreads + t]: a warp's 16-byte reads of one
+// slot are contiguous.
+constexpr int kStageSlots = 2 * kDigestUnroll;                       // 16-byte words per thread per stage
+constexpr uint32_t kStageBytes = 2u * kStageSlots * kThreads * 16u;  // two stages: 73,728 bytes
+
+__device__ __forceinline__ void cp16(uint32_t dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_wait_all_but_newest() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
 __device__ __forceinline__ void flush(uint64_t &acc, int slot, unsigned long long *s_acc) {
   uint64_t x = acc;
 #pragma unroll
@@ -139,13 +162,15 @@ __device__ __forceinline__ uint32_t word_at(const DigestEntry &E, uint64_t i) {
                       : (uint32_t) reinterpret_cast<const uint16_t *>(E.data)[i];
 }
 
-// Two CTAs per SM (24 warps).  The bound lets the compiler use 80 registers:
-// without per-vector checks a full tile's 24 terms form one block that it
-// schedules for more overlap than 64 registers hold.
+// Two CTAs per SM (24 warps, 2 x 72 KB of stages).  The bound lets the
+// compiler use 80 registers: without per-vector checks a full tile's 24 terms
+// form one block that it schedules for more overlap than 64 registers hold.
 template <int MAXE>
 __global__ void __launch_bounds__(kThreads, 2) digest_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
                                                           unsigned long long *out) {
   __shared__ unsigned long long s_acc[APC_MAX_SLOTS];
+  extern __shared__ __align__(16) uint4 stg[];
+  const uint32_t stg_t = (uint32_t)__cvta_generic_to_shared(stg + threadIdx.x);  // this thread's slot 0, stage 0
   if (threadIdx.x < APC_MAX_SLOTS) s_acc[threadIdx.x] = 0;
   __syncthreads();
   const uint32_t one = plan.one;
@@ -182,8 +207,33 @@ __global__ void __launch_bounds__(kThreads, 2) digest_kernel(const __grid_consta
     if (E.dtype == 0) {
       const uint32_t *d = reinterpret_cast<const uint32_t *>(E.data);
       const uint4 *q = reinterpret_cast<const uint4 *>(d + base);
-      for (; tile < full_end; ++tile, q += kDigestTile / 4, G0 += (uint32_t)kDigestTile)
-        tile32(q, all, G0, one, t0, t1);
+      if (tile < full_end) {
+        uint32_t b = 0;
+#pragma unroll
+        for (int k = 0; k < kStageSlots; ++k) cp16(stg_t + k * kThreads * 16u, q + (k >> 1) * 2 * kThreads + (k & 1));
+        cp_commit();
+        for (; tile < full_end; ++tile, q += kDigestTile / 4, G0 += (uint32_t)kDigestTile) {
+          if (tile + 1 < full_end) {
+            const uint4 *n = q + kDigestTile / 4;
+            const uint32_t dst = stg_t + (b ^ 1) * kStageSlots * kThreads * 16u;
+#pragma unroll
+            for (int k = 0; k < kStageSlots; ++k) cp16(dst + k * kThreads * 16u, n + (k >> 1) * 2 * kThreads + (k & 1));
+          }
+          cp_commit();
+          cp_wait_all_but_newest();
+          const uint4 *src = stg + b * kStageSlots * kThreads + threadIdx.x;
+          uint4 x[kDigestUnroll][2];
+#pragma unroll
+          for (int u = 0; u < kDigestUnroll; ++u) {
+            x[u][0] = src[(2 * u) * kThreads];
+            x[u][1] = src[(2 * u + 1) * kThreads];
+          }
+          const uint32_t B = G0 + 0x9E3779B9u;
+          if (top_bits_shared(B, kTileKeySpan)) fold32<true>(x, all, G0, one, B >> 30, t0, t1);
+          else fold32<false>(x, all, G0, one, 0, t0, t1);
+          b ^= 1;
+        }
+      }
       if (tile < stop) {  // the entry's last tile
         last_tile_ok((uint64_t)(reinterpret_cast<const uint32_t *>(q) - d), vec_end, ok);
         tile32(q, ok, G0, one, t0, t1);
@@ -192,8 +242,30 @@ __global__ void __launch_bounds__(kThreads, 2) digest_kernel(const __grid_consta
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
       const uint4 *q = reinterpret_cast<const uint4 *>(d + base);
-      for (; tile < full_end; ++tile, q += kDigestTile / 8, G0 += (uint32_t)kDigestTile)
-        tile16(q, all, G0, one, t0, t1);
+      if (tile < full_end) {
+        uint32_t b = 0;
+#pragma unroll
+        for (int u = 0; u < kDigestUnroll; ++u) cp16(stg_t + u * kThreads * 16u, q + u * kThreads);
+        cp_commit();
+        for (; tile < full_end; ++tile, q += kDigestTile / 8, G0 += (uint32_t)kDigestTile) {
+          if (tile + 1 < full_end) {
+            const uint4 *n = q + kDigestTile / 8;
+            const uint32_t dst = stg_t + (b ^ 1) * kStageSlots * kThreads * 16u;
+#pragma unroll
+            for (int u = 0; u < kDigestUnroll; ++u) cp16(dst + u * kThreads * 16u, n + u * kThreads);
+          }
+          cp_commit();
+          cp_wait_all_but_newest();
+          const uint4 *src = stg + b * kStageSlots * kThreads + threadIdx.x;
+          uint4 x[kDigestUnroll];
+#pragma unroll
+          for (int u = 0; u < kDigestUnroll; ++u) x[u] = src[u * kThreads];
+          const uint32_t B = G0 + 0x9E3779B9u;
+          if (top_bits_shared(B, kTileKeySpan)) fold16<true>(x, all, G0, one, B >> 30, t0, t1);
+          else fold16<false>(x, all, G0, one, 0, t0, t1);
+          b ^= 1;
+        }
+      }
       if (tile < stop) {  // the entry's last tile
         last_tile_ok((uint64_t)(reinterpret_cast<const uint16_t *>(q) - d), vec_end, ok);
         tile16(q, ok, G0, one, t0, t1);
@@ -218,22 +290,49 @@ __global__ void __launch_bounds__(kThreads, 2) digest_kernel(const __grid_consta
 
 }  // namespace
 
+namespace {
+// The dynamic shared-memory limit of one instantiation, raised once per
+// device (later launches, for example inside a stream capture, only enqueue).
+template <int MAXE>
+int ensure_stage_attribute() {
+  static std::atomic<uint64_t> done_mask{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return (int)e;
+  const uint64_t bit = dev < 64 ? (1ull << dev) : 0;
+  if (bit && (done_mask.load(std::memory_order_acquire) & bit)) return 0;
+  e = cudaFuncSetAttribute(digest_kernel<MAXE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStageBytes);
+  if (e != cudaSuccess) return (int)e;
+  if (bit) done_mask.fetch_or(bit, std::memory_order_acq_rel);
+  return 0;
+}
+
+template <int MAXE>
+int launch_t(const DigestPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
+  int e = ensure_stage_attribute<MAXE>();
+  if (e) return e;
+  digest_kernel<MAXE><<<grid, kThreads, kStageBytes, (cudaStream_t)stream>>>(plan, out);
+  return (int)cudaGetLastError();
+}
+
+template <int MAXE>
+int blocks_t(int *out) {
+  int e = ensure_stage_attribute<MAXE>();
+  if (e) return e;
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<MAXE>, kThreads, kStageBytes);
+}
+}  // namespace
+
 int launch_digest_small(const DigestPlan<kDigestSmall> &plan, unsigned grid, void *stream,
                         unsigned long long *out) {
-  digest_kernel<kDigestSmall><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
-  return (int)cudaGetLastError();
+  return launch_t<kDigestSmall>(plan, grid, stream, out);
 }
 
 int launch_digest_large(const DigestPlan<kDigestLarge> &plan, unsigned grid, void *stream,
                         unsigned long long *out) {
-  digest_kernel<kDigestLarge><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
-  return (int)cudaGetLastError();
+  return launch_t<kDigestLarge>(plan, grid, stream, out);
 }
 
-int digest_blocks_per_sm(bool large, int *out) {
-  cudaError_t e = large ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<kDigestLarge>, kThreads, 0)
-                        : cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<kDigestSmall>, kThreads, 0);
-  return (int)e;
-}
+int digest_blocks_per_sm(bool large, int *out) { return large ? blocks_t<kDigestLarge>(out) : blocks_t<kDigestSmall>(out); }
 
 }  // namespace apc
