@@ -288,9 +288,6 @@ __global__ void __launch_bounds__(kThreads, 2) digest_kernel(const __grid_consta
   if (threadIdx.x < APC_MAX_SLOTS && s_acc[threadIdx.x]) atomicAdd(&out[threadIdx.x], s_acc[threadIdx.x]);
 }
 
-}  // namespace
-
-namespace {
 // The dynamic shared-memory limit of one instantiation, raised once per
 // device (later launches, for example inside a stream capture, only enqueue).
 template <int MAXE>
@@ -321,6 +318,7 @@ int blocks_t(int *out) {
   if (e) return e;
   return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<MAXE>, kThreads, kStageBytes);
 }
+
 }  // namespace
 
 int launch_digest_small(const DigestPlan<kDigestSmall> &plan, unsigned grid, void *stream,
