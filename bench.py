@@ -45,6 +45,12 @@ FALLBACK_HBM_GBS = 6800.0
 # ----------------------------------------------------------------- helpers
 
 L2_BYTES = 129 << 20          # the GB300's L2
+# Integer-ALU ceiling of the verification pass: 152 SMs x 4 sub-partitions x
+# 16 ALU lanes at the 2.07 GHz maximum SM clock, over the pass's integer-ALU
+# instructions per splitmix64 term (ncu instruction count and ALU pipe
+# utilisation of digest_kernel on the 152M-element case).
+ALU_LANE_OPS_PER_S = 152 * 64 * 2.07e9
+VERIFY_ALU_INSTRUCTIONS_PER_TERM = 13.1
 
 # What each synthetic workload stands for (synth/workloads.py).
 WORKLOAD_TEXT = {
@@ -90,7 +96,8 @@ def kernel_source_hash(kernel: str) -> str:
 
 
 def profiled_traffic(kernel: str, workload: str):
-    """DRAM bytes per launch of ``kernel`` from the committed ncu summary,
+    """DRAM bytes of one launch (the commit) or one pass (the verification,
+    whatever its launch count) of ``kernel`` from the committed ncu summary,
     if it was taken on the current kernel sources; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
@@ -102,7 +109,7 @@ def profiled_traffic(kernel: str, workload: str):
         return None
     if rec.get("workload") != workload:
         return None
-    return rec.get("dram_bytes_per_launch")
+    return rec.get("dram_bytes_per_launch", rec.get("dram_bytes_per_pass"))
 
 
 class ClockSampler:
@@ -617,6 +624,7 @@ def run_gpu(args):
     c_ms = statistics.median(commit_ms)
     v_ms = statistics.median(verify_ms)
     c_avg = sum(commit_ms) / K
+    v_avg = sum(verify_ms) / K
     achieved = COMMIT_BYTES * N / (c_avg * 1e-3) / 1e9
     line = {
         "metric": METRIC,
@@ -649,6 +657,15 @@ def run_gpu(args):
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": profiled_traffic("commit_kernel", w.name),
                      "algorithmic_bytes_per_launch": COMMIT_BYTES * N},
+        "roofline_verify": {"bound": "alu", "kernel": "digest_kernel", "achieved": 4 * N / (v_avg * 1e-3) / 1e12,
+                            "peak": ALU_LANE_OPS_PER_S / VERIFY_ALU_INSTRUCTIONS_PER_TERM / 1e12,
+                            "unit": "T splitmix64 terms/s",
+                            "frac": 4 * N / (v_avg * 1e-3) / (ALU_LANE_OPS_PER_S / VERIFY_ALU_INSTRUCTIONS_PER_TERM),
+                            "peak_basis": "152 SMs x 64 integer-ALU lanes x 2.07 GHz over %.1f ALU instructions "
+                                          "per term" % VERIFY_ALU_INSTRUCTIONS_PER_TERM,
+                            "launches": n_digest_launches,
+                            "traffic": profiled_traffic("digest_kernel", w.name),
+                            "algorithmic_bytes": VERIFY_BYTES * N},
         "gpu_launches": K * (n_commit_launches + n_digest_launches),
         "gpu_launches_note": "per timed step: %d commit_kernel + %d digest_kernel launches (%d tensors, %d buffers; "
                              "up to 440 tensors and 1000 buffers per launch)"
