@@ -14,18 +14,19 @@
 // Warp-specialized pipeline (one persistent CTA per SM by default):
 //  * The producer warp walks the launch's tiles (L::kTile elements of one
 //    entry's 16-byte aligned body: 4,864 for fp32 state, 9,728 for bf16
-//    state) and, for each, waits until a ring
-//    stage is free and issues four bulk asynchronous copies -- p, m, v and g
-//    -- that complete on the stage's "full" mbarrier.  Loads never occupy
-//    consumer registers, and up to kCommitStages tiles per CTA are in flight.
+//    state) and, for each, waits until a ring stage is free and issues four
+//    bulk asynchronous copies -- p, m, v and g -- that complete on the
+//    stage's "full" mbarrier.  Loads never occupy consumer registers, and up
+//    to kCommitStages tiles per CTA are in flight.
 //  * With each stage the producer also writes a 48-byte descriptor (the
 //    tile's first-element addresses in p, m, v, w, g, its element count and
 //    first digest index) into shared memory before arming the stage, so the
 //    consumers never search the chunk table themselves.
 //  * The consumer warps (19 by default) wait for a stage, read its
 //    descriptor and their elements from shared memory (thread t of C takes
-//    elements 4t..4t+3 and 4C+4t..4C+4t+3, so both the shared-memory reads
-//    and the global stores are contiguous across the warp), release the
+//    the groups 4kC+4t..4kC+4t+3 for k < L::kGroups, 2 for fp32 state and 4
+//    for bf16 state, so both the shared-memory reads and the global stores
+//    are contiguous across the warp), release the
 //    stage to the producer, then apply AdamW, store the results with
 //    streaming stores, and fold the digest terms into 64-bit registers.
 //  * Elements outside the aligned bodies (entry heads and tails under 8
