@@ -13,7 +13,7 @@
 //
 // Warp-specialized pipeline (one persistent CTA per SM by default):
 //  * The producer warp walks the launch's tiles (L::kTile elements of one
-//    entry's 16-byte aligned body: 4,864 for fp32 state, 9,728 for bf16
+//    entry's 16-byte aligned body: 4,864 for fp32 state, 10,368 for bf16
 //    state) and, for each, waits until a ring stage is free and issues four
 //    bulk asynchronous copies -- p, m, v and g -- that complete on the
 //    stage's "full" mbarrier.  Loads never occupy consumer registers, and up
@@ -22,11 +22,11 @@
 //    tile's first-element addresses in p, m, v, w, g, its element count and
 //    first digest index) into shared memory before arming the stage, so the
 //    consumers never search the chunk table themselves.
-//  * The consumer warps (19 by default) wait for a stage, read its
-//    descriptor and their elements from shared memory (thread t of C takes
-//    the groups 4kC+4t..4kC+4t+3 for k < L::kGroups, 2 for fp32 state and 4
-//    for bf16 state, so both the shared-memory reads and the global stores
-//    are contiguous across the warp), release the
+//  * The consumer warps (19 for fp32 state, 27 for bf16 state) wait for a
+//    stage, read its descriptor and their elements from shared memory
+//    (thread t of C takes the groups 4kC+4t..4kC+4t+3 for k < L::kGroups, 2
+//    for fp32 state and 3 for bf16 state, so both the shared-memory reads and
+//    the global stores are contiguous across the warp), release the
 //    stage to the producer, then apply AdamW, store the results with
 //    streaming stores, and fold the digest terms into 64-bit registers.
 //  * Elements outside the aligned bodies (entry heads and tails under 8
@@ -84,7 +84,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 // A consumer thread's output addresses in the current tile: element
 // start + 4t of the entry (t the consumer index).  Group k of the thread then
-// sits at a compile-time element offset k * 4 * kCommitConsumers, which the
+// sits at a compile-time element offset k * 4 * L::kConsumers, which the
 // stores carry as an immediate.
 struct Dst {
   void *p, *m, *v;
@@ -125,6 +125,9 @@ __device__ __forceinline__ uint64_t hterm(uint32_t G, uint32_t bits, uint32_t on
 struct F32State {
   static constexpr uint32_t kES = 4;        // bytes per state element
   static constexpr int kDigests = 4;
+  static constexpr int kConsumerWarps = kCommitConsumerWarps;
+  static constexpr int kConsumers = 32 * kConsumerWarps;
+  static constexpr int kThreads = kConsumers + 32;  // + the producer warp
   static constexpr int kGroups = kCommitGroups;
   static constexpr uint64_t kTile = kCommitTile;
   struct Regs {
@@ -201,6 +204,9 @@ struct F32State {
 struct BF16State {
   static constexpr uint32_t kES = 2;
   static constexpr int kDigests = 3;
+  static constexpr int kConsumerWarps = kCommitConsumerWarpsBF16;
+  static constexpr int kConsumers = 32 * kConsumerWarps;
+  static constexpr int kThreads = kConsumers + 32;
   static constexpr int kGroups = kCommitGroupsBF16;
   static constexpr uint64_t kTile = kCommitTileBF16;
   struct Regs {
@@ -273,13 +279,13 @@ struct BF16State {
 };
 
 // Group K of a consumer thread's tile: its elements sit at the compile-time
-// offset K * 4 * kCommitConsumers from the thread's output addresses, which
+// offset K * 4 * L::kConsumers from the thread's output addresses, which
 // the stores carry as immediates and the digest terms fold into their
 // increment.
 template <class L, bool ZERO, int K>
 __device__ __forceinline__ void store_groups(const Dst &d, uint32_t G1, const typename L::Regs *r, const bool *ok,
                                              const Scalars &s, Acc &a) {
-  constexpr uint32_t off = (uint32_t)(K * kCommitConsumers) * 4;
+  constexpr uint32_t off = (uint32_t)(K * L::kConsumers) * 4;
   if (ok[K]) {
     if (ZERO) __stcs(reinterpret_cast<uint2 *>(d.g + off), make_uint2(0u, 0u));
     L::template compute_store<off>(d, G1, r[K], s, a);
@@ -306,20 +312,20 @@ __device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint
 }
 
 template <class L, int MAXE, bool ZERO>
-__global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
+__global__ void __launch_bounds__(L::kThreads, kCommitBlocksPerSm)
     commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan, unsigned long long *out) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ __align__(8) uint64_t full[kCommitStages];
   __shared__ __align__(8) uint64_t empty[kCommitStages];
   __shared__ StageDesc desc[kCommitStages];
-  __shared__ uint64_t red[kCommitThreads / 32];
+  __shared__ uint64_t red[L::kThreads / 32];
   __shared__ int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kCommitStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], kCommitConsumerWarps);
+      mbar_init(&empty[s], L::kConsumerWarps);
     }
     abort_flag = 0;
     mbar_init_fence();
@@ -327,7 +333,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
   __syncthreads();
 
   Acc a{0, 0, 0, 0};
-  if (warp == kCommitConsumerWarps) {
+  if (warp == L::kConsumerWarps) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       const uint64_t policy = l2_evict_first();
@@ -381,7 +387,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
   } else {
     // ----------------------------------------------------------- consumers
     const Scalars s{plan.h, plan.one};
-    const int ct = threadIdx.x;  // 0 .. kCommitConsumers-1
+    const int ct = threadIdx.x;  // 0 .. L::kConsumers-1
     uint32_t phase = 0;
     int stage = 0;
     for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
@@ -396,7 +402,7 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
       bool ok[L::kGroups];
 #pragma unroll
       for (int k = 0; k < L::kGroups; ++k) {
-        const uint32_t e = (uint32_t)(k * kCommitConsumers + ct) * 4;
+        const uint32_t e = (uint32_t)(k * L::kConsumers + ct) * 4;
         ok[k] = e < sd.cnt;
         if (ok[k]) L::load(st, e, r[k]);
       }
@@ -415,8 +421,8 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
     // scalar items: entry heads and tails, and entries without vectors
     if (!*(volatile int *)&abort_flag) {
       uint32_t cur = 0;
-      for (uint64_t it = (uint64_t)blockIdx.x * kCommitConsumers + ct; it < plan.total_scalar;
-           it += (uint64_t)gridDim.x * kCommitConsumers) {
+      for (uint64_t it = (uint64_t)blockIdx.x * L::kConsumers + ct; it < plan.total_scalar;
+           it += (uint64_t)gridDim.x * L::kConsumers) {
         while (cur + 1 < plan.count && it >= plan.e[cur + 1].scalar_begin) ++cur;
         const CommitEntry &E = plan.e[cur];
         const uint64_t k = it - E.scalar_begin;
@@ -435,14 +441,14 @@ __global__ void __launch_bounds__(kCommitThreads, kCommitBlocksPerSm)
 
   const bool ok = !*(volatile int *)&abort_flag;
   uint64_t r;
-  r = cta_sum<kCommitThreads>(a.p, red);
+  r = cta_sum<L::kThreads>(a.p, red);
   if (threadIdx.x == 0 && ok && r) atomicAdd(&out[0], (unsigned long long)r);
-  r = cta_sum<kCommitThreads>(a.m, red);
+  r = cta_sum<L::kThreads>(a.m, red);
   if (threadIdx.x == 0 && ok && r) atomicAdd(&out[1], (unsigned long long)r);
-  r = cta_sum<kCommitThreads>(a.v, red);
+  r = cta_sum<L::kThreads>(a.v, red);
   if (threadIdx.x == 0 && ok && r) atomicAdd(&out[2], (unsigned long long)r);
   if (L::kDigests == 4) {
-    r = cta_sum<kCommitThreads>(a.w, red);
+    r = cta_sum<L::kThreads>(a.w, red);
     if (threadIdx.x == 0 && ok && r) atomicAdd(&out[3], (unsigned long long)r);
   }
 }
@@ -478,7 +484,7 @@ template <class L, int MAXE, bool ZERO>
 int launch_t(const CommitPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
   int e = ensure_smem_attribute<L, MAXE, ZERO>();
   if (e) return e;
-  commit_kernel<L, MAXE, ZERO><<<grid, kCommitThreads, smem_bytes<L>(), (cudaStream_t)stream>>>(plan, out);
+  commit_kernel<L, MAXE, ZERO><<<grid, L::kThreads, smem_bytes<L>(), (cudaStream_t)stream>>>(plan, out);
   return (int)cudaGetLastError();
 }
 
@@ -496,7 +502,7 @@ template <class L, int MAXE>
 int blocks_per_sm(int *out) {
   int e = ensure_smem_attribute<L, MAXE, false>();
   if (e) return e;
-  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<L, MAXE, false>, kCommitThreads,
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, commit_kernel<L, MAXE, false>, L::kThreads,
                                                             smem_bytes<L>());
 }
 

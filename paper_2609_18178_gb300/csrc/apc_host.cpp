@@ -169,7 +169,8 @@ apc_status run_commit_batches(const std::vector<apc::CommitEntry> &entries, cons
     plan->count = (uint32_t)k;
     plan->total_tiles = tiles;
     plan->total_scalar = scalars;
-    const uint64_t want = std::max<uint64_t>(tiles, (scalars + apc::kCommitConsumers - 1) / apc::kCommitConsumers);
+    const uint64_t consumers = (uint64_t)apc::commit_consumers(layout);
+    const uint64_t want = std::max<uint64_t>(tiles, (scalars + consumers - 1) / consumers);
     const unsigned grid = (unsigned)std::max<uint64_t>(1, std::min<uint64_t>(want, grid_cap));
     int e = launch(*plan, layout, zero_grad, grid, stream, out);
     if (e) return cuda_fail(e, "commit kernel launch");

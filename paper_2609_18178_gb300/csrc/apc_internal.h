@@ -15,22 +15,33 @@ constexpr uint32_t kScalarMode = 0xFFFFFFFFu;  // `head` value of an entry run w
 
 // Commit kernel: warp-specialized pipeline.  One producer warp streams each
 // tile of p, m, v and g into a ring of shared-memory stages with bulk
-// asynchronous copies; kCommitConsumerWarps warps compute from shared memory
-// and store straight to global memory.
+// asynchronous copies; the consumer warps compute from shared memory and
+// store straight to global memory.
 //
-// Pipeline shape (compile-time; the defaults are the measured best on GB300).
-// 19 consumer warps + 1 producer = 20 warps, 5 per SM sub-partition: each
-// sub-partition's 16,384 registers then give 96 per thread with no spills,
-// the same budget as 16 + 1 warps (whose fifth warp on one sub-partition sets
-// the cap), with three more warps issuing.
+// Pipeline shape (compile-time, per state layout; the defaults are the
+// measured best on GB300).
+//  * fp32 state: 19 consumer warps + 1 producer = 20 warps, 5 per SM
+//    sub-partition: each sub-partition's 16,384 registers then give 96 per
+//    thread with no spills, the same budget as 16 + 1 warps (whose fifth
+//    warp on one sub-partition sets the cap), with three more warps issuing.
+//    Each consumer thread takes 2 groups of 4 elements per tile (3 ran 6%
+//    slower).
+//  * bf16 state stages 8 bytes per element instead of 14 and needs fewer
+//    registers: 27 consumer warps + 1 producer = 28 warps at 72 registers
+//    with no spills, 3 groups per thread per tile.  That is 3.2% faster than
+//    the fp32 layout's shape there (19 warps and 4 groups were 1.8% faster
+//    than 19 and 2; 23 warps with 3 groups and 31 with 2 were in between).
 #ifndef APC_COMMIT_CONSUMER_WARPS
 #define APC_COMMIT_CONSUMER_WARPS 19
+#endif
+#ifndef APC_COMMIT_CONSUMER_WARPS_BF16
+#define APC_COMMIT_CONSUMER_WARPS_BF16 27
 #endif
 #ifndef APC_COMMIT_GROUPS
 #define APC_COMMIT_GROUPS 2
 #endif
 #ifndef APC_COMMIT_GROUPS_BF16
-#define APC_COMMIT_GROUPS_BF16 4
+#define APC_COMMIT_GROUPS_BF16 3
 #endif
 #ifndef APC_COMMIT_STAGES
 #define APC_COMMIT_STAGES 2
@@ -39,26 +50,24 @@ constexpr uint32_t kScalarMode = 0xFFFFFFFFu;  // `head` value of an entry run w
 #define APC_COMMIT_BLOCKS_PER_SM 1
 #endif
 constexpr int kCommitConsumerWarps = APC_COMMIT_CONSUMER_WARPS;
-constexpr int kCommitConsumers = kCommitConsumerWarps * 32;
-constexpr int kCommitThreads = kCommitConsumers + 32;                   // + the producer warp
-// 4-element groups per consumer thread per tile, for each state layout.  The
-// bf16 layout, with half the staged bytes per element, takes 4 (1.8% faster
-// than 2 there; 3 gave 1.2%, 5 was slower); the fp32 layout keeps 2 (3 ran
-// 6% slower).
+constexpr int kCommitConsumerWarpsBF16 = APC_COMMIT_CONSUMER_WARPS_BF16;
 constexpr int kCommitGroups = APC_COMMIT_GROUPS;
 constexpr int kCommitGroupsBF16 = APC_COMMIT_GROUPS_BF16;
-constexpr uint64_t kCommitTile = (uint64_t)kCommitConsumers * 4 * kCommitGroups;          // 4,864 elements
-constexpr uint64_t kCommitTileBF16 = (uint64_t)kCommitConsumers * 4 * kCommitGroupsBF16;  // 9,728 elements
+constexpr uint64_t kCommitTile = (uint64_t)kCommitConsumerWarps * 32 * 4 * kCommitGroups;              // 4,864 elements
+constexpr uint64_t kCommitTileBF16 = (uint64_t)kCommitConsumerWarpsBF16 * 32 * 4 * kCommitGroupsBF16;  // 10,368 elements
 constexpr int kCommitStages = APC_COMMIT_STAGES;
 constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
 // A stage holds one tile of p, m, v and g: 14 bytes per element for fp32
-// state (133 KB per CTA at the defaults), 8 for bf16 state (152 KB).
+// state (133 KB per CTA at the defaults), 8 for bf16 state (162 KB).
 
 // State layouts of the commit kernel.
 constexpr int kLayoutF32 = 0;   // fp32 p, m, v; bf16 g; bf16 copy w
 constexpr int kLayoutBF16 = 1;  // bf16 p, m, v; bf16 g; no copy
 
 constexpr uint64_t commit_tile(int layout) { return layout == kLayoutBF16 ? kCommitTileBF16 : kCommitTile; }
+constexpr int commit_consumers(int layout) {
+  return 32 * (layout == kLayoutBF16 ? kCommitConsumerWarpsBF16 : kCommitConsumerWarps);
+}
 
 // One chunk-table entry of the commit kernel (72 bytes).
 //   p, m, v: fp32 or bf16 state (by the launch's layout); w: the bf16 copy

@@ -588,8 +588,8 @@ def run_bf16(tensors, step, hp=HP, zero_grad=False, shift=0):
     assert apc.digests_to_host(out) == want
 
 
-# Elements per tile of the commit kernel's bf16-state layout (19 x 32 threads x 4 groups of 4).
-COMMIT_TILE_BF16 = 9728
+# Elements per tile of the commit kernel's bf16-state layout (27 x 32 threads x 3 groups of 4).
+COMMIT_TILE_BF16 = 10368
 
 
 @pytest.mark.parametrize("n", [1, 3, 7, 8, 9, 63, 4864, 4871, 9728 + 5, 100003] +
