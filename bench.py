@@ -759,7 +759,8 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["c1", "c2", "c3", "c4", "c5"], default="c5")
-    ap.add_argument("--e2e-steps", type=int, default=8)
+    ap.add_argument("--e2e-steps", type=int, default=16,
+                    help="timed end-to-end steps (each timed region starts with an empty upload pipeline)")
     ap.add_argument("--e2e-groups", type=int, default=12)
     ap.add_argument("--f3-tensors", type=int, default=0,
                     help="next row f3 over the first K tensors of its shard only (0 = all; for profiling)")
