@@ -51,9 +51,9 @@ __device__ __forceinline__ uint32_t adamw_element(float &p, float &m, float &v, 
 // faster depends on the kernel around it (both give the same bits):
 //  * MulWide: three multiply-adds, lo*clo widened, then lo*chi and hi*clo
 //    added into the high word.  Fewest instructions; the commit kernel,
-//    which is bound by instruction issue, runs 3% faster with it.
+//    which is bound by instruction issue, runs 2.7% faster with it.
 //  * MulCompiler: the compiler's own 64-bit multiply.  The verification
-//    pass, which is bound by the integer ALU rather than by issue, runs 2.5%
+//    pass, which is bound by the integer ALU rather than by issue, runs 3.3%
 //    faster with it.
 struct MulWide {
   template <uint32_t CLO, uint32_t CHI>
