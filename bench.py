@@ -684,6 +684,26 @@ def run_gpu(args):
 
 # --------------------------------------------------------- CPU oracle arm
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the architecture)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.machine()
+
+
 def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
     """The oracle (as it stands) on all host cores over a bounded sample: the
     first ``sample`` elements of the workload's flat order, one step = the
@@ -722,7 +742,7 @@ def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
         el = time.perf_counter() - t0
         if el >= seconds or el * (done + n) / done > 3 * seconds:
             break
-    return {"value": done / el, "unit": "elements/s", "cores": cores, "kind": "oracle",
+    return {"value": done / el, "unit": "elements/s", "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
             "sample": "first %d elements of %s (embed_tokens), step %d (commit + verification digests), "
                       "%d passes, %.1f s" % (n, w.name, step_t, done // n, el),
             "verify_matches_commit": ok}
