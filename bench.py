@@ -716,6 +716,7 @@ def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
     n = min(sample, w.n)
     cores = os.cpu_count() or 1
     g0 = w.pieces[0].goff
+    where = w.pieces[0].name if n <= w.pieces[0].n else "from %s on" % w.pieces[0].name
     p, m, v = synth.state(n, g0)
     g = synth.grad(n, g0, step_t)
     h8 = oracle.resolve_hparams(HP, step_t)
@@ -743,8 +744,8 @@ def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
         if el >= seconds or el * (done + n) / done > 3 * seconds:
             break
     return {"value": done / el, "unit": "elements/s", "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
-            "sample": "first %d elements of %s (embed_tokens), step %d (commit + verification digests), "
-                      "%d passes, %.1f s" % (n, w.name, step_t, done // n, el),
+            "sample": "first %d elements of %s (%s), step %d (commit + verification digests), "
+                      "%d passes, %.1f s" % (n, w.name, where, step_t, done // n, el),
             "verify_matches_commit": ok}
 
 
