@@ -519,9 +519,14 @@ int launch_commit_large(const CommitPlan<kCommitLarge> &plan, int layout, bool z
 }
 
 int commit_blocks_per_sm(bool large, int *out) {
-  // the fp32 layout has the larger shared-memory footprint, so its residency
-  // also holds for the bf16 layout
-  return large ? blocks_per_sm<F32State, kCommitLarge>(out) : blocks_per_sm<F32State, kCommitSmall>(out);
+  // one grid size serves both layouts: the smaller of their residencies
+  int f = 0, b = 0;
+  int e = large ? blocks_per_sm<F32State, kCommitLarge>(&f) : blocks_per_sm<F32State, kCommitSmall>(&f);
+  if (e) return e;
+  e = large ? blocks_per_sm<BF16State, kCommitLarge>(&b) : blocks_per_sm<BF16State, kCommitSmall>(&b);
+  if (e) return e;
+  *out = f < b ? f : b;
+  return 0;
 }
 
 int launch_wait_timeout(uint64_t limit_ns, void *stream) {
