@@ -41,7 +41,11 @@
  *            elements apart have equal keys.
  *
  * Conventions for every call:
- *   - Device pointers belong to the calling thread's current CUDA device.
+ *   - Device pointers belong to the calling thread's current CUDA device:
+ *     every buffer a kernel reads or writes, and every output, must be
+ *     device memory of that device (or managed memory).  Each call checks
+ *     this with one cudaPointerGetAttributes query per distinct address and
+ *     returns APC_EINVAL for host memory or another device's memory.
  *     The caller owns all memory and the library allocates nothing.  Between
  *     calls it keeps only each device's SM count and kernel residency
  *     (queried once), the kernels' device status word (apc_device_status)
@@ -75,7 +79,7 @@ typedef struct CUstream_st *apc_stream_t;
 typedef enum apc_status {
   APC_OK = 0,
   APC_EINVAL = 1, /* null pointer, bad count, out-of-range hyper-parameter or step,
-                     overlapping outputs                                          */
+                     overlapping outputs, memory that is not the current device's */
   APC_EALIGN = 2, /* pointer not aligned to its element size                       */
   APC_ERANGE = 3, /* global_offset + n overflows 64 bits                           */
   APC_ECUDA = 4,  /* the CUDA runtime reported an error (launch or attribute query) */
@@ -123,15 +127,23 @@ typedef struct apc_buffer {
 
 /* The committed AdamW step plus state digest over a chunk table.
  *
+ * Defines the step that reaches the committed optimizer boundary (arxiv
+ * 2609.18178 Section I; Section III-C, phase 2): it updates the preserved
+ * state W, M, V of S_app for optimizer step tau_opt (Section III-A, Eq. 2)
+ * and emits the digests that the bitwise rank-state checks compare
+ * (Sections IV-F, IV-G).
+ *
  * table[0..num_tensors): the tensors of one rank's shard (any number; tables
  *   larger than one launch's capacity are split into several launches on
  *   `stream`, with identical results).  num_tensors == 0 is valid.
  * hp, step: hyper-parameters and the 1-based optimizer step t (tau_opt).
  * out_digests: device, 4 x uint64, written as {D_p', D_m', D_v', D_w}; it is
- *   zeroed on `stream` first, so it need not be initialised.
+ *   zeroed on `stream` first, so it need not be initialised.  It must not
+ *   overlap any buffer of the table.
  * Returns APC_EINVAL (null table with num_tensors > 0, null hp or
  * out_digests, num_tensors < 0, step < 1, hyper-parameters out of range,
- * overlapping outputs), APC_EALIGN, APC_ERANGE, APC_ECUDA, or APC_OK. */
+ * overlapping outputs, a buffer or out_digests that is not memory of the
+ * current device), APC_EALIGN, APC_ERANGE, APC_ECUDA, or APC_OK. */
 apc_status apc_commit_step(const apc_tensor *table, int32_t num_tensors, const apc_adamw_hparams *hp,
                            int64_t step, apc_stream_t stream, uint64_t *out_digests);
 
@@ -173,13 +185,19 @@ apc_status apc_commit_step_bf16(const apc_tensor_bf16 *table, int32_t num_tensor
 
 /* The state digest of a list of buffers, read only.
  *
+ * The post-recovery verification: peers compare these digests to prove
+ * that device state is bit-identical without checkpoint I/O (the bitwise
+ * rank-state checks of arxiv 2609.18178, Abstract and Sections IV-F, IV-G,
+ * over the preserved W, M, V of Section III-A, Eq. 2).
+ *
  * bufs[0..num_bufs): buffers; each adds its elements into out_digests[slot].
  * num_slots: 1..APC_MAX_SLOTS; out_digests (device, num_slots x uint64) is
- *   zeroed on `stream` first.
+ *   zeroed on `stream` first; it must not overlap any buffer of the list.
  * The digest of the four buffers that apc_commit_step wrote, given as slots
  * 0..3 with the table's offsets, equals that call's out_digests.
  * Returns APC_EINVAL (null pointers, bad counts, bad dtype, slot >=
- * num_slots), APC_EALIGN, APC_ERANGE, APC_ECUDA, or APC_OK. */
+ * num_slots, an output that overlaps a buffer, a pointer that is not memory
+ * of the current device), APC_EALIGN, APC_ERANGE, APC_ECUDA, or APC_OK. */
 apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, apc_stream_t stream,
                       uint64_t *out_digests);
 
@@ -194,7 +212,9 @@ apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs, int32_t n
 
 /* The eight binary32 scalars that apc_commit_step passes to the device for
  * step t, in the order b1, 1-b1, b2, 1-b2, eps, 1-lr*wd, lr/(1-b1^t),
- * 1/sqrt(1-b2^t).  Host only; no CUDA call.  out: host, 8 floats. */
+ * 1/sqrt(1-b2^t).  t is the optimizer step tau_opt of the preserved state
+ * (arxiv 2609.18178 Section III-A, Eq. 2), on which the bias corrections
+ * depend.  Host only; no CUDA call.  out: host, 8 floats. */
 apc_status apc_resolve_hparams(const apc_adamw_hparams *hp, int64_t step, float out[8]);
 
 /* One segment of apc_upload: `bytes` bytes from `src` to `dst`.
@@ -237,10 +257,22 @@ apc_status apc_set_reserved_sms(int32_t n);
 
 /* Device-side status of this library's kernels on the current device since
  * the previous call: APC_OK, or APC_ETIMEOUT if a bounded wait inside a
- * kernel gave up (the digests and updates of that launch are then incomplete;
- * a kernel that gives up stops, drains its own copies and exits, leaving the
- * context usable).  Synchronizes the device, reads the status word and clears
- * it.  Returns APC_ECUDA if the CUDA runtime reports an error. */
+ * kernel gave up.  A kernel that gives up stops, drains its own copies and
+ * exits, leaving the context usable, but its work is incomplete:
+ *   - after apc_commit_step(_ex, _bf16), the shard is torn: some tiles hold
+ *     step t and others step t-1, in place, and the launch's digests are
+ *     dropped.  Nothing in the library can roll it back.  The shard must be
+ *     restored from a replica (or checkpoint) before training continues:
+ *     the fail-stop rule of the recovery protocol (arxiv 2609.18178 Section
+ *     III-C, safety invariant).
+ *   - after apc_digest or apc_count_nonzero, only the outputs are wrong; the
+ *     call can be repeated.
+ * A wait gives up after at least 2^20 polls and 1 s of the GPU's global
+ * timer; a kernel that is descheduled does not poll, so time slicing alone
+ * does not make it give up, but a GPU shared with other contexts can in
+ * principle delay a healthy wait past the limit.
+ * Synchronizes the device, reads the status word and clears it.  Returns
+ * APC_ECUDA if the CUDA runtime reports an error. */
 apc_status apc_device_status(void);
 
 /* Self-test of the bounded-wait path: launch one thread on `stream` that

@@ -130,14 +130,21 @@ def _hp(hp: dict | None) -> _HParams:
 
 
 def _ptr(x, itemsize: int | None = None) -> int:
-    """Device address of a torch tensor (checked: CUDA, contiguous, element
-    size) or a raw integer pointer."""
+    """Device address of a torch tensor (checked: on the current CUDA device,
+    contiguous, element size) or a raw integer pointer.  The library launches
+    on the calling thread's current device, so a tensor of another device is
+    refused here rather than dereferenced there."""
     if x is None:
         return 0
     if isinstance(x, int):
         return x
     if not x.is_cuda:
         raise ValueError("tensor is not on a CUDA device")
+    import torch
+    cur = torch.cuda.current_device()
+    if x.device.index != cur:
+        raise ValueError("tensor is on cuda:%s but the current device is cuda:%d (use torch.cuda.device(...))"
+                         % (x.device.index, cur))
     if not x.is_contiguous():
         raise ValueError("tensor is not contiguous")
     if itemsize is not None and x.element_size() != itemsize:

@@ -144,6 +144,49 @@ unsigned grid_for(uint64_t tiles, int sms, int per_sm) {
   return (unsigned)std::max<uint64_t>(1, std::min(tiles, cap));
 }
 
+// A pointer that a kernel will dereference, with what it is for the error
+// message: `list` ("table", "bufs", "out"), entry index and field name.
+struct Owned {
+  const void *p;
+  const char *list;
+  int index;
+  const char *field;
+};
+
+// Every buffer a kernel reads or writes must be memory of the calling
+// thread's current device (or managed memory): a pointer into another GPU's
+// memory, or host memory, would otherwise be dereferenced by this device's
+// copies.  One attribute query per distinct address.  Returns APC_ECUDA if
+// the runtime cannot answer (for example, no device) and APC_EINVAL naming the
+// first foreign pointer (lowest address first).
+apc_status check_device_pointers(std::vector<Owned> &ptrs) {
+  if (ptrs.empty()) return APC_OK;
+  int dev = 0;
+  int e = (int)cudaGetDevice(&dev);
+  if (e) return cuda_fail(e, "cudaGetDevice");
+  std::sort(ptrs.begin(), ptrs.end(), [](const Owned &a, const Owned &b) { return a.p < b.p; });
+  const void *last = nullptr;
+  for (const Owned &o : ptrs) {
+    if (o.p == last) continue;
+    last = o.p;
+    cudaPointerAttributes a;
+    e = (int)cudaPointerGetAttributes(&a, o.p);
+    if (e) {
+      cudaGetLastError();  // clear the runtime's error state of the failed query
+      return cuda_fail(e, "cudaPointerGetAttributes");
+    }
+    const bool own = (a.type == cudaMemoryTypeDevice && a.device == dev) || a.type == cudaMemoryTypeManaged;
+    if (!own) {
+      if (o.index >= 0)
+        return fail(APC_EINVAL, "%s[%d].%s is not memory of the current device %d (memory type %d, device %d)",
+                    o.list, o.index, o.field, dev, (int)a.type, a.device);
+      return fail(APC_EINVAL, "%s is not memory of the current device %d (memory type %d, device %d)", o.list, dev,
+                  (int)a.type, a.device);
+    }
+  }
+  return APC_OK;
+}
+
 // Entries arrive with their tile count in tile_begin and their scalar-item
 // count in scalar_begin; each batch turns both into prefix offsets.
 template <int MAXE, typename Launch>
@@ -240,8 +283,10 @@ apc_status commit_common(int layout, const std::vector<TableRow> &rows, const ap
 
   std::vector<apc::CommitEntry> entries;
   std::vector<Range> ranges;
+  std::vector<Owned> owned;
   entries.reserve(rows.size());
-  ranges.reserve(rows.size() * 5);
+  ranges.reserve(rows.size() * 5 + 1);
+  owned.reserve(rows.size() * 5 + 1);
   for (size_t k = 0; k < rows.size(); ++k) {
     const TableRow &t = rows[k];
     if (t.n == 0) continue;
@@ -259,6 +304,12 @@ apc_status commit_common(int layout, const std::vector<TableRow> &rows, const ap
     ranges.push_back({v, v + es * t.n, true});
     if (t.w) ranges.push_back({w, w + 2 * t.n, true});
     ranges.push_back({g, g + 2 * t.n, zero_grad});
+    const int ki = (int)k;
+    owned.push_back({t.p, "table", ki, "p"});
+    owned.push_back({t.m, "table", ki, "m"});
+    owned.push_back({t.v, "table", ki, "v"});
+    owned.push_back({t.g, "table", ki, "g"});
+    if (t.w) owned.push_back({t.w, "table", ki, "w"});
     // first element at which all buffers sit on a 16-byte boundary
     const uint64_t h0 = ((16 - g % 16) % 16) / 2;
     const bool aligned = (p + es * h0) % 16 == 0 && (m + es * h0) % 16 == 0 && (v + es * h0) % 16 == 0 &&
@@ -284,7 +335,12 @@ apc_status commit_common(int layout, const std::vector<TableRow> &rows, const ap
     }
     entries.push_back(e);
   }
-  if (overlaps(ranges)) return fail(APC_EINVAL, "table buffers overlap (a written range meets another range)");
+  const uintptr_t o = (uintptr_t)out_digests;
+  ranges.push_back({o, o + (uintptr_t)nslots * sizeof(uint64_t), true});
+  if (overlaps(ranges))
+    return fail(APC_EINVAL, "table buffers or out_digests overlap (a written range meets another range)");
+  owned.push_back({out_digests, "out_digests", -1, ""});
+  if ((st = check_device_pointers(owned)) != APC_OK) return st;
 
   int e = (int)cudaMemsetAsync(out_digests, 0, (size_t)nslots * sizeof(uint64_t), (cudaStream_t)stream);
   if (e) return cuda_fail(e, "cudaMemsetAsync(out_digests)");
@@ -346,6 +402,10 @@ apc_status buffer_entries(const apc_buffer *bufs, int32_t num_bufs, int32_t num_
   if (!out) return fail(APC_EINVAL, "output pointer is null");
   if ((uintptr_t)out % 8) return fail(APC_EALIGN, "output not 8-byte aligned");
   entries->reserve((size_t)num_bufs);
+  std::vector<Range> ranges;
+  std::vector<Owned> owned;
+  ranges.reserve((size_t)num_bufs + 1);
+  owned.reserve((size_t)num_bufs + 1);
   for (int32_t k = 0; k < num_bufs; ++k) {
     const apc_buffer &b = bufs[k];
     if (b.dtype != APC_F32 && b.dtype != APC_BF16) return fail(APC_EINVAL, "bufs[%d]: unknown dtype %u", k, b.dtype);
@@ -357,6 +417,8 @@ apc_status buffer_entries(const apc_buffer *bufs, int32_t num_bufs, int32_t num_
     const uintptr_t a = (uintptr_t)b.data;
     const uint64_t es = b.dtype == APC_F32 ? 4 : 2;
     if (a % es) return fail(APC_EALIGN, "bufs[%d]: data not %u-byte aligned", k, (unsigned)es);
+    ranges.push_back({a, a + es * b.n, false});
+    owned.push_back({b.data, "bufs", (int)k, "data"});
     apc::DigestEntry e;
     e.data = b.data;
     e.n = b.n;
@@ -369,7 +431,11 @@ apc_status buffer_entries(const apc_buffer *bufs, int32_t num_bufs, int32_t num_
     e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kDigestTile));  // tile count until placed
     entries->push_back(e);
   }
-  return APC_OK;
+  const uintptr_t o = (uintptr_t)out;
+  ranges.push_back({o, o + (uintptr_t)num_slots * sizeof(uint64_t), true});
+  if (overlaps(ranges)) return fail(APC_EINVAL, "the output overlaps a buffer of the list");
+  owned.push_back({out, "output", -1, ""});
+  return check_device_pointers(owned);
 }
 
 }  // namespace

@@ -52,7 +52,7 @@ def _locked_build(target: str, sources: list[str], cmd_for) -> None:
 
 def build_host() -> str:
     _locked_build(_HOST_SO, [_SRC_H, _SRC_HOST], lambda out: [
-        "gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
+        "gcc", "-O3", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
         "-pthread", "-fvisibility=hidden", _SRC_HOST, "-o", out])
     return _HOST_SO
 

@@ -113,19 +113,39 @@ def oracle_at(gidx: np.ndarray, step: int, hp=None):
     return dict(p=p.view(np.uint32), m=m.view(np.uint32), v=v.view(np.uint32), w=w)
 
 
-def oracle_workload_digest(w: W.Workload, step: int, hp=None, chunk: int = 1 << 24):
+def oracle_workload_digest(w: W.Workload, step: int, hp=None, chunk: int = 1 << 22, workers: int | None = None,
+                           inspect=None):
     """The four digests of one step over a workload from the generated state,
-    streamed through the oracle chunk by chunk (host memory stays bounded)."""
+    streamed through the oracle chunk by chunk (host memory stays bounded).
+
+    Chunks run concurrently on ``workers`` threads (default: every host
+    core), each generating its inputs and running the oracle single-threaded;
+    the oracle and the generator are C calls that release the GIL.  The
+    digests of the chunks are added mod 2^64, which is the digest of their
+    concatenation.  ``inspect(piece, start, outputs)``, if given, is called
+    (on a worker thread) for every chunk of every piece with
+    ``outputs = dict(p, m, v, w)`` holding the oracle's written bits of
+    elements [start, start + n) of that piece, so that a test can compare
+    whole tensors element by element on the way."""
+    from concurrent.futures import ThreadPoolExecutor
     hp = hp or oracle.DEFAULT_HP
     h8 = oracle.resolve_hparams(hp, step)
+    jobs = [(pc, s) for pc in w.pieces for s in range(0, pc.n, chunk)]
+
+    def run(job):
+        pc, s = job
+        n = min(chunk, pc.n - s)
+        g0 = pc.goff + s
+        p, m, v = synth.state(n, g0, nthreads=1)
+        g = synth.grad(n, g0, step, nthreads=1)
+        wb, d = oracle.commit(p, m, v, g, g0, h8, nthreads=1)
+        if inspect is not None:
+            inspect(pc, s, dict(p=p.view(np.uint32), m=m.view(np.uint32), v=v.view(np.uint32), w=wb))
+        return d
+
     tot = [0, 0, 0, 0]
-    for pc in w.pieces:
-        for s in range(0, pc.n, chunk):
-            n = min(chunk, pc.n - s)
-            g0 = pc.goff + s
-            p, m, v = synth.state(n, g0, nthreads=NTHREADS)
-            g = synth.grad(n, g0, step, nthreads=NTHREADS)
-            _, d = oracle.commit(p, m, v, g, g0, h8, nthreads=NTHREADS)
+    with ThreadPoolExecutor(workers or NTHREADS) as ex:
+        for d in ex.map(run, jobs):
             tot = [(a + b) & M64 for a, b in zip(tot, d)]
     return tot
 

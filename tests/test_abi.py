@@ -146,9 +146,54 @@ def _no_device():
 
 
 def test_valid_call_without_device_reports_cuda_error():
+    """A call that passes argument validation next asks the runtime which
+    device owns each pointer; without a device that query fails and the call
+    returns APC_ECUDA before anything is enqueued."""
     _no_device()
     assert commit([fake(8)]) == 4
-    assert apc.library().apc_last_error().startswith(b"cudaMemsetAsync")
+    assert apc.library().apc_last_error().startswith((b"cudaGetDevice", b"cudaPointerGetAttributes"))
+
+
+def test_outputs_overlapping_inputs_are_rejected():
+    """out_digests (commit) and the output of apc_digest / apc_count_nonzero
+    are written ranges: meeting any buffer of the call is APC_EINVAL, found
+    on the host before any CUDA call."""
+    lib = apc.library()
+    assert commit([fake(100)], out=BASE + 64) == 1                       # inside p
+    assert commit([fake(100)], out=BASE + (3 << 30) + 8) == 1            # inside the gradient
+    assert commit([fake(100)], out=BASE + (4 << 30) + 192) == 1          # inside w (200 bytes)
+    assert b"out_digests" in lib.apc_last_error()
+
+    def dig(fn, bufs, slots, out):
+        arr = (_B * max(1, len(bufs)))(*bufs)
+        return fn(ctypes.addressof(arr), len(bufs), slots, None, ctypes.c_void_p(out))
+
+    for fn in (lib.apc_digest, lib.apc_count_nonzero):
+        assert dig(fn, [_B(BASE, 16, 0, 0, 0)], 1, BASE + 56) == 1       # last 8 bytes of 64
+        assert dig(fn, [_B(BASE, 16, 0, 0, 0)], 4, BASE - 24) == 1      # slots 3 meets the buffer
+        assert b"overlaps" in lib.apc_last_error()
+
+
+def test_binding_refuses_a_tensor_of_another_device(monkeypatch):
+    """The binding passes only tensors of the current device to the library."""
+    torch = pytest.importorskip("torch")
+
+    class Fake:
+        is_cuda = True
+        device = torch.device("cuda", 1)
+
+        def is_contiguous(self):
+            return True
+
+        def element_size(self):
+            return 4
+
+        def data_ptr(self):
+            return BASE
+
+    monkeypatch.setattr(torch.cuda, "current_device", lambda: 0)
+    with pytest.raises(ValueError, match="current device"):
+        apc._ptr(Fake(), 4)
 
 
 def test_shared_gradient_is_not_an_overlap():

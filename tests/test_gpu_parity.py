@@ -373,12 +373,26 @@ def test_c4_rank_shard_pieces_equal_one_entry():
     assert da == oracle_workload_digest(wp, 5)
 
 
+# Whole tensors of every shape class of Mistral-7B, compared element by
+# element on the way through the streamed oracle of the full model.
+C5_WHOLE_TENSORS = ("embed_tokens", "layers.13.q_proj", "layers.13.k_proj", "layers.20.down_proj",
+                    "layers.31.post_attention_layernorm", "norm", "lm_head")
+
+
 def test_c5_full_model_bench_configuration():
     """The benchmark's workload: all 291 Mistral-7B tensors (7,248,023,552
     elements) in separate allocations, step 18, the same table and launch
-    configuration as bench.py.  Sampled elements against the oracle; the
-    verify pass equals the fused digests; the 16 rank shards' digests sum to
-    the whole (concatenation)."""
+    configuration as bench.py.
+
+    The whole state is checked against the oracle: the four digests of
+    p', m', v', w equal those of the oracle streamed over every element of
+    the model (the bitwise rank-state check of Sections IV-F/IV-G over the
+    W, M, V of Section III-A, Eq. 2), and whole tensors of each shape class
+    (embedding, q, k, down projections, both RMSNorm kinds, lm_head) equal it
+    bit for bit.  The verify pass equals the fused digests, and the 16 rank
+    shards' digests sum to the whole (concatenation)."""
+    import threading
+    import time
     w = W.c5()
     free, total = torch.cuda.mem_get_info()
     if free < 130 * (1 << 30):
@@ -400,6 +414,35 @@ def test_c5_full_model_bench_configuration():
         d = apc.digests_to_host(apc.digest(bufs, 4))
         total = [(x + y) & M64 for x, y in zip(total, d)]
     assert total == got
+    torch.cuda.synchronize()
+
+    names = set(C5_WHOLE_TENSORS)
+    assert names <= {pc.name for pc in w.pieces}
+    compared, bad, lock = {}, [], threading.Lock()
+
+    def inspect(pc, start, ref):
+        if pc.name not in names:
+            return
+        B = dw.bufs[pc.alloc]
+        n = len(ref["w"])
+        sl = slice(pc.at + start, pc.at + start + n)
+        for k in "pmv":
+            dev_bits = B[k][sl].cpu().numpy().view(np.uint32)
+            if not np.array_equal(dev_bits, ref[k]):
+                with lock:
+                    bad.append((pc.name, k, start, int(np.count_nonzero(dev_bits != ref[k]))))
+        if not np.array_equal(B["w"][sl].cpu().numpy().view(np.uint16), ref["w"]):
+            with lock:
+                bad.append((pc.name, "w", start))
+        with lock:
+            compared[pc.name] = compared.get(pc.name, 0) + n
+
+    t0 = time.perf_counter()
+    want = oracle_workload_digest(w, 18, inspect=inspect)
+    print("c5 oracle stream: %d elements in %.1f s" % (w.n, time.perf_counter() - t0))
+    assert not bad, bad[:5]
+    assert compared == {pc.name: pc.n for pc in w.pieces if pc.name in names}
+    assert got == want
     del dw
     torch.cuda.empty_cache()
 
