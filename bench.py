@@ -11,9 +11,13 @@ than L2 (129 MB), so no flush is needed between timed steps.
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
 a bounded sample of the same workload instead.
 
-Multi-GPU (torchrun): rank r commits its own shard -- a full-size copy of
-the workload's table at global offset r * N, so the job's flat model is the
-concatenation of the ranks' shards and per-GPU work is fixed (weak scaling).
+Multi-GPU (torchrun), two partitions (--split):
+  copy   (default) rank r commits a full-size copy of the workload's table at
+         global offset r * N, so the job's flat model is the concatenation of
+         the ranks' copies and per-GPU work is fixed (weak scaling);
+  model  rank r commits the contiguous range r of the one model's flat
+         parameters (the flat-parameter partition of FSDP), so total work is
+         fixed (strong scaling).
 There is no collective on the data path.  A Gloo control plane brackets the
 timed region with barriers, takes the maximum time over ranks, and after
 timing gathers every rank's digests (the whole-model digest is their
@@ -218,6 +222,19 @@ def exchange_digests(dist, step: int, commit_digests: list[int], verify_digests:
     return ag.whole_digests, True
 
 
+def sum_over_ranks(dist, digests: list[int]) -> list[int]:
+    """Digests added over the ranks mod 2^64 (the whole model's, by
+    concatenation): a control-plane all-reduce of int64 bit patterns, whose
+    sum wraps exactly as the unsigned sum does."""
+    d = [int(x) & M64 for x in digests]
+    if dist is None:
+        return d
+    import torch
+    t = torch.tensor([x - (1 << 64) if x >= 1 << 63 else x for x in d], dtype=torch.int64)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return [int(x) & M64 for x in t.tolist()]
+
+
 def group_pieces(sizes: list[int], n_groups: int) -> list[list[int]]:
     """Consecutive runs of table entries with about equal element counts."""
     total = sum(sizes)
@@ -347,10 +364,19 @@ def run_gpu(args):
     dist = init_control_plane(world)
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = W.ALL[args.workload]()
-    step_t = w.steps[-1]
+    whole = W.ALL[args.workload]()
+    step_t = whole.steps[-1]
+    if args.split == "model":
+        # flat-parameter partition: rank r commits the contiguous range r of
+        # the one model (total work fixed as ranks are added)
+        w = W.shard(whole, rank, world)
+        base, N_job = 0, whole.n
+    else:
+        # every rank commits a full-size copy at global offset r * N: the
+        # job's flat model is the concatenation of the copies
+        w = whole
+        base, N_job = shard_offset(rank, whole.n), world * whole.n
     N = w.n
-    base = shard_offset(rank, N)   # this rank's shard of the job's flat model
 
     # resident state: one allocation per tensor, filled by the device generator
     stream = torch.cuda.current_stream()
@@ -381,6 +407,10 @@ def run_gpu(args):
     # would: no Python work sits between a timed event and its launch
     tab, vtab = apc.prepare_table(entries), apc.prepare_buffers(vbufs)
     torch.cuda.synchronize()
+    # The first commit runs from the generated state, the same step the
+    # oracle computes from the same generated inputs in cpu_baseline's c5
+    # stream; later steps update the state in place.
+    first_digests = apc.digests_to_host(apc.commit_step(tab, step_t, HP, stream=s, out=out_c))
 
     def one_step(ev=None):
         if ev is not None:
@@ -413,7 +443,8 @@ def run_gpu(args):
     ms_per_step = total_ms / K
     digests_c = apc.digests_to_host(out_c)
     digests_v = apc.digests_to_host(out_v)
-    whole, verified = exchange_digests(dist, step_t, digests_c, digests_v, shard=rank)
+    whole_d, verified = exchange_digests(dist, step_t, digests_c, digests_v, shard=rank)
+    first_whole = sum_over_ranks(dist, first_digests)
 
     # End to end: every step brings its gradient from pinned host memory and
     # returns the digests.  The table is cut into groups of about equal size;
@@ -526,7 +557,7 @@ def run_gpu(args):
 
         h2d_ms = upload_alone(use_sm)
         ce_ms = upload_alone(False) if use_sm else h2d_ms
-        e2e = {"value": world * N / (e2e_ms * 1e-3), "unit": "elements/s",
+        e2e = {"value": N_job / (e2e_ms * 1e-3), "unit": "elements/s",
                "h2d_bytes_per_step": 2 * N, "d2h_bytes_per_step": 64 * n_groups, "ms_per_step": e2e_ms,
                "steps": ke, "groups": n_groups, "verify_matches_commit": e2e_verified,
                "upload": ({"method": "apc_upload: SM loads of pinned host memory over the host link",
@@ -602,9 +633,9 @@ def run_gpu(args):
                                           "frac": 2 * N / (guard_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 2,
                                           "nonzero_before": nz_before, "nonzero_after_zeroing": nz_after}}
 
-    cpu = None
+    cpu, oracle_c5 = None, None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w, step_t, args.cpu_seconds)
+        cpu, oracle_c5 = cpu_baseline(os.cpu_count() or 1, plan_c5=args.cpu_plan == "full")
 
     if rank == 0 and world == 1 and not args.no_next and args.replicas > 1:
         # the c5 state stays resident (116 GB); the replicas add 4 x 7.3 GB
@@ -628,21 +659,25 @@ def run_gpu(args):
     achieved = COMMIT_BYTES * N / (c_avg * 1e-3) / 1e9
     line = {
         "metric": METRIC,
-        "value": world * N / (ms_per_step * 1e-3),
+        "value": N_job / (ms_per_step * 1e-3),
         "unit": "elements/s",
         "n_gpus": world,
         "steps": K,
         "warmup": args.warmup,
         "ms_per_step": ms_per_step,
         "higher_is_better": True,
-        "scaling": "weak",
+        "scaling": "strong" if args.split == "model" else "weak",
         "vs_baseline": None,
         "dtype": "f32+u64",
         "data": "synthetic",
         "config": {"workload": "%s: %s, %d tensors, %d elements, step %d, commit+digest then re-verify"
-                               % (w.name, WORKLOAD_TEXT.get(w.name, "synthetic shard"), len(w.pieces), N, step_t),
-                   "elements": N, "tensors": len(w.pieces), "step": step_t,
-                   "parallelism": "%d ranks x one shard each (no data-path collective)" % world,
+                               % (whole.name, WORKLOAD_TEXT.get(whole.name, "synthetic shard"), len(whole.pieces),
+                                  whole.n, step_t),
+                   "elements": N_job, "elements_per_rank": N, "tensors": len(whole.pieces), "step": step_t,
+                   "split": args.split,
+                   "parallelism": ("%d ranks x one contiguous range of the flat model each (no data-path "
+                                   "collective)" % world if args.split == "model" else
+                                   "%d ranks x one full-size shard each (no data-path collective)" % world),
                    "l2": ("inputs larger than L2 (%.1f GB resident state)" % (16 * N / 1e9)
                           if COMMIT_BYTES * N > L2_BYTES else
                           "inputs smaller than L2 (%.3f GB per step): timings include L2 hits" % (COMMIT_BYTES * N / 1e9))},
@@ -670,7 +705,15 @@ def run_gpu(args):
         "gpu_launches_note": "per timed step: %d commit_kernel + %d digest_kernel launches (%d tensors, %d buffers; "
                              "up to 440 tensors and 1000 buffers per launch)"
                              % (n_commit_launches, n_digest_launches, len(entries), len(vbufs)),
-        "digests": ["%016x" % d for d in whole],
+        "digests": ["%016x" % d for d in whole_d],
+        "first_commit_digests": ["%016x" % d for d in first_whole],
+        "oracle_parity": (None if oracle_c5 is None or w.name != "c5" or world != 1 else
+                          {"workload": "c5", "step": step_t,
+                           "gpu_first_commit_digests": ["%016x" % d for d in first_digests],
+                           "oracle_digests": ["%016x" % d for d in oracle_c5],
+                           "equal": first_digests == oracle_c5,
+                           "what": "digests of p', m', v', w after one step from the generated state: the GPU's "
+                                   "first (untimed) commit against the oracle streamed over every element"}),
         "verify_matches_commit": verified,
         "clocks": clk,
         "e2e": e2e,
@@ -704,72 +747,161 @@ def cpu_model() -> str:
     return platform.machine()
 
 
-def cpu_baseline(w, step_t: int, seconds: float, sample: int = 1 << 26):
-    """The oracle (as it stands) on all host cores over a bounded sample: the
-    first ``sample`` elements of the workload's flat order, one step = the
-    oracle's commit (threaded) then its digests of the four written buffers
-    (the verification pass, chunks on a thread pool), repeated until
-    ``seconds`` of work; input generation is not timed."""
-    from concurrent.futures import ThreadPoolExecutor
+def _oracle_step(p, m, v, g, g0: int, h8, threads: int, pool=None):
+    """One oracle step over the contiguous global range [g0, g0 + n): the
+    committed step (the oracle's own threaded partition when threads > 1),
+    then the verification digests of the four written buffers (chunks on
+    ``pool`` when threads > 1).  Updates p, m, v in place.  Returns
+    (commit seconds, verify seconds, commit digests, verification matches)."""
     import oracle
-    import synth
-    n = min(sample, w.n)
-    cores = os.cpu_count() or 1
-    g0 = w.pieces[0].goff
-    where = w.pieces[0].name if n <= w.pieces[0].n else "from %s on" % w.pieces[0].name
-    p, m, v = synth.state(n, g0)
-    g = synth.grad(n, g0, step_t)
-    h8 = oracle.resolve_hparams(HP, step_t)
-    chunk = -(-n // cores)
-
-    def verify(wb):
+    n = p.size
+    t0 = time.perf_counter()
+    wb, d = oracle.commit(p, m, v, g, g0, h8, nthreads=threads)
+    t1 = time.perf_counter()
+    if threads <= 1 or pool is None:
+        dv = [oracle.digest_f32(p, g0), oracle.digest_f32(m, g0), oracle.digest_f32(v, g0), oracle.digest_u16(wb, g0)]
+    else:
+        chunk = -(-n // threads)
         parts = []
         for lo in range(0, n, chunk):
             hi = min(n, lo + chunk)
             parts += [(oracle.digest_f32, p[lo:hi], lo), (oracle.digest_f32, m[lo:hi], lo),
                       (oracle.digest_f32, v[lo:hi], lo), (oracle.digest_u16, wb[lo:hi], lo)]
-        with ThreadPoolExecutor(cores) as ex:
-            res = list(ex.map(lambda a: a[0](a[1], g0 + a[2]), parts))
-        tot = [0, 0, 0, 0]
-        for k, r in enumerate(res):
-            tot[k % 4] = (tot[k % 4] + r) & M64
-        return tot
+        dv = [0, 0, 0, 0]
+        for k, r in enumerate(pool.map(lambda a: a[0](a[1], g0 + a[2]), parts)):
+            dv[k % 4] = (dv[k % 4] + r) & M64
+    t2 = time.perf_counter()
+    return t1 - t0, t2 - t1, d, d == dv
 
-    done, ok, t0 = 0, True, time.perf_counter()
-    while True:
-        wb, d = oracle.commit(p, m, v, g, g0, h8, nthreads=cores)
-        ok = ok and verify(wb) == d
-        done += n
-        el = time.perf_counter() - t0
-        if el >= seconds or el * (done + n) / done > 3 * seconds:
-            break
-    return {"value": done / el, "unit": "elements/s", "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
-            "sample": "first %d elements of %s (%s), step %d (commit + verification digests), "
-                      "%d passes, %.1f s" % (n, w.name, where, step_t, done // n, el),
-            "verify_matches_commit": ok}
+
+def _flat_range(w):
+    """The workload's global index range; every workload's pieces cover one
+    contiguous range, so the oracle can run it as one flat shard (the digest
+    of a concatenation is the sum of the digests, so the table's split does
+    not change any result)."""
+    lo = min(pc.goff for pc in w.pieces)
+    hi = max(pc.goff + pc.n for pc in w.pieces)
+    assert hi - lo == w.n
+    return lo, hi
+
+
+def cpu_baseline(cores: int, plan_c5: bool = True, chunk: int = 1 << 22):
+    """The oracle (as it stands) on the host cores, per the measurement plan:
+    c2, c3 and c4 each timed single-threaded and on all cores over the whole
+    workload, and c5 streamed over all of its elements in chunks on all
+    cores, with each chunk's oracle compute timed on its own thread (input
+    generation is not timed).  One step = the committed step plus the
+    verification digests of the written buffers.  Returns the record and the
+    oracle's c5 digests of one step from the generated state."""
+    from concurrent.futures import ThreadPoolExecutor
+    import oracle
+    import synth
+    from synth import workloads as W
+    configs = {}
+    with ThreadPoolExecutor(cores) as pool:
+        for name in ("c2", "c3", "c4"):
+            w = W.ALL[name]()
+            lo, hi = _flat_range(w)
+            step = w.steps[-1]
+            h8 = oracle.resolve_hparams(HP, step)
+            p, m, v = synth.state(hi - lo, lo, nthreads=cores)
+            g = synth.grad(hi - lo, lo, step, nthreads=cores)
+            rec = {"elements": w.n, "step": step}
+            for label, th in (("single_thread", 1), ("all_cores", cores)):
+                cs, vs, _, ok = _oracle_step(p, m, v, g, lo, h8, th, pool)
+                rec[label] = {"threads": th, "commit_s": cs, "verify_s": vs,
+                              "elements_per_s": w.n / (cs + vs), "verify_matches_commit": ok}
+            configs[name] = rec
+            del p, m, v, g
+    c5_digests = None
+    if plan_c5:
+        w = W.c5()
+        step = w.steps[-1]
+        h8 = oracle.resolve_hparams(HP, step)
+        lo, hi = _flat_range(w)
+
+        def one(start):
+            n = min(chunk, hi - start)
+            p, m, v = synth.state(n, start, nthreads=1)
+            g = synth.grad(n, start, step, nthreads=1)
+            cs, vs, d, ok = _oracle_step(p, m, v, g, start, h8, 1)
+            return cs, vs, d, ok
+
+        t0 = time.perf_counter()
+        cs_sum = vs_sum = 0.0
+        tot, ok_all, nchunks = [0, 0, 0, 0], True, 0
+        with ThreadPoolExecutor(cores) as pool:
+            for cs, vs, d, ok in pool.map(one, range(lo, hi, chunk)):
+                cs_sum += cs
+                vs_sum += vs
+                tot = [(a + b) & M64 for a, b in zip(tot, d)]
+                ok_all = ok_all and ok
+                nchunks += 1
+        wall = time.perf_counter() - t0
+        c5_digests = tot
+        configs["c5"] = {"elements": w.n, "step": step, "chunks": nchunks, "chunk_elements": chunk,
+                         "threads": cores, "commit_cpu_s": cs_sum, "verify_cpu_s": vs_sum,
+                         "elements_per_s_per_core": w.n / (cs_sum + vs_sum),
+                         "elements_per_s_all_cores": w.n * cores / (cs_sum + vs_sum),
+                         "wall_s_with_generation": wall, "verify_matches_commit": ok_all,
+                         "digests": ["%016x" % x for x in tot],
+                         "note": "sum over chunks of each chunk's oracle compute on its own thread; all cores "
+                                 "= elements x threads / summed compute seconds"}
+    if "c5" in configs:
+        value, sample = configs["c5"]["elements_per_s_all_cores"], (
+            "all %d elements of c5 (step 18) in %d chunks of %d on %d threads; commit + verification digests; "
+            "value = elements x threads / summed per-chunk compute seconds; input generation not timed"
+            % (configs["c5"]["elements"], configs["c5"]["chunks"], chunk, cores))
+    else:
+        value, sample = configs["c4"]["all_cores"]["elements_per_s"], (
+            "all %d elements of c4 (step 5) on %d threads, commit + verification digests" % (W.c4().n, cores))
+    rec = {"value": value, "unit": "elements/s", "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
+           "sample": sample, "configs": configs}
+    return rec, c5_digests
 
 
 def run_reference(args):
+    """The reference arm: the CPU oracle as it stands, on the host cores.
+    Each step is one oracle step (commit + verification digests, on all
+    cores) over a bounded sample of the workload: its first
+    --ref-elements elements; ms_per_step and value are measured on exactly
+    those elements."""
     world, rank, _ = dist_env()
     if rank != 0:
         return
+    from concurrent.futures import ThreadPoolExecutor
+    import oracle
+    import synth
     from synth import workloads as W
     w = W.ALL[args.workload]()
     step_t = w.steps[-1]
-    # each "step" is a bounded sample of the workload on the host cores
-    per_step = max(1.0, args.cpu_seconds / max(1, args.steps + args.warmup))
-    for _ in range(args.warmup):
-        cpu_baseline(w, step_t, per_step)
-    vals = [cpu_baseline(w, step_t, per_step) for _ in range(args.steps)]
-    v = statistics.median(x["value"] for x in vals)
-    cb = dict(vals[0], value=v)
-    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "elements/s", "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * w.n / v, "higher_is_better": True,
+    lo, hi = _flat_range(w)
+    n = min(args.ref_elements, hi - lo)
+    cores = os.cpu_count() or 1
+    h8 = oracle.resolve_hparams(HP, step_t)
+    p, m, v = synth.state(n, lo, nthreads=cores)
+    g = synth.grad(n, lo, step_t, nthreads=cores)
+    times, ok = [], True
+    with ThreadPoolExecutor(cores) as pool:
+        for k in range(args.warmup + args.steps):
+            cs, vs, _, good = _oracle_step(p, m, v, g, lo, h8, cores, pool)
+            ok = ok and good
+            if k >= args.warmup:
+                times.append(cs + vs)
+    t = sum(times) / len(times)
+    v_ = n / t
+    first = w.pieces[0].name
+    sample = ("first %d of the %d elements of %s (from %s on), step %d, committed step + verification digests "
+              "on %d threads, %d timed steps" % (n, w.n, w.name, first, step_t, cores, len(times)))
+    line = {"impl": "reference", "metric": METRIC, "value": v_, "unit": "elements/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32+u64", "data": "synthetic",
-            "config": {"workload": "%s (CPU oracle on a bounded sample)" % w.name, "elements": w.n,
-                       "step": step_t},
-            "cpu_baseline": cb,
-            "e2e": {"value": v, "unit": "elements/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+            "config": {"workload": "%s: CPU oracle over a bounded sample (%s)" % (w.name, sample), "elements": n,
+                       "workload_elements": w.n, "step": step_t},
+            "verify_matches_commit": ok,
+            "cpu_baseline": {"value": v_, "unit": "elements/s", "cores": cores, "cpu_model": cpu_model(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": v_, "unit": "elements/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
@@ -780,6 +912,9 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["c1", "c2", "c3", "c4", "c5"], default="c5")
+    ap.add_argument("--split", choices=["copy", "model"], default="copy",
+                    help="multi-GPU: every rank a full-size copy of the workload (copy, weak scaling) or rank r "
+                         "the contiguous range r of the one model's flat parameters (model, strong scaling)")
     ap.add_argument("--e2e-steps", type=int, default=16,
                     help="timed end-to-end steps (each timed region starts with an empty upload pipeline)")
     ap.add_argument("--e2e-groups", type=int, default=12)
@@ -789,7 +924,11 @@ def main(argv=None):
                     help="end-to-end upload: apc_upload on a few CTAs, or the DMA copy engines")
     ap.add_argument("--e2e-upload-ctas", type=int, default=16)
     ap.add_argument("--e2e-reserved-sms", type=int, default=8)
-    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--ref-elements", type=int, default=1 << 28,
+                    help="reference arm: oracle elements per step (a bounded sample of the workload)")
+    ap.add_argument("--cpu-plan", choices=["full", "configs"], default="full",
+                    help="cpu_baseline: c2-c4 single-thread and all-core, plus c5 streamed over every element "
+                         "(full), or c2-c4 only (configs)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")

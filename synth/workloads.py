@@ -151,4 +151,23 @@ def f3(rank: int = 1, world: int = 4) -> Workload:
     return w
 
 
+def shard(w: Workload, rank: int, world: int) -> Workload:
+    """Rank ``rank``'s part of a workload under a flat-parameter (FSDP)
+    partition: the contiguous range [N*r/world, N*(r+1)/world) of the
+    workload's flat index range, cut from its pieces.  Each cut piece keeps
+    its own allocation, of just its elements, and its global offset, so the
+    digests of the ranks' shards add up to the workload's (Section II-A:
+    every rank holds one contiguous range of the flattened parameters)."""
+    lo0 = min(p.goff for p in w.pieces)
+    lo, hi = rank_range(rank, world, w.n)
+    lo, hi = lo0 + lo, lo0 + hi
+    pieces, allocs = [], []
+    for p in w.pieces:
+        a, b = max(p.goff, lo), min(p.goff + p.n, hi)
+        if a < b:
+            pieces.append(Piece(p.name, b - a, a, alloc=len(allocs), at=0))
+            allocs.append(b - a)
+    return Workload("%s[%d/%d]" % (w.name, rank, world), pieces, list(w.steps), w.chained, w.verify, allocs)
+
+
 ALL = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5}
