@@ -49,12 +49,54 @@ FALLBACK_HBM_GBS = 6800.0
 # ----------------------------------------------------------------- helpers
 
 L2_BYTES = 129 << 20          # the GB300's L2
-# Integer-ALU ceiling of the verification pass: 152 SMs x 4 sub-partitions x
-# 16 ALU lanes at the 2.07 GHz maximum SM clock, over the pass's integer-ALU
-# instructions per splitmix64 term (ncu instruction count and ALU pipe
-# utilisation of digest_kernel on the 152M-element case).
-ALU_LANE_OPS_PER_S = 152 * 64 * 2.07e9
-VERIFY_ALU_INSTRUCTIONS_PER_TERM = 13.1
+# The verification pass's work per splitmix64 term, counted from the
+# definition (first output of SplitMix64 seeded with the key, summed mod
+# 2^64) in 32-bit operations:
+#   increment            64-bit add                          2 adds
+#   z ^= z >> 30, 27, 31 per xor-shift: a funnel shift for the low half, a
+#                        shift for the high half, two xors    3 x (1 + 1 + 2)
+#   z *= C1, C2          per multiply: low x low widened, the two cross
+#                        products into the high word         2 x 3 multiply-adds
+#   D += z               64-bit add (one three-input add per half for a pair
+#                        of terms)                           1 add
+# minus what two identities remove: the high half's first shift is one per
+# run of keys whose incremented high words share their top two bits (the
+# kernels check this per tile); for a 16-bit word the increment never carries
+# and leaves the low half's top bits at 01, so the first funnel shift is the
+# single multiply-add 4*hi + 1.  Where the operations can run:
+#   xors                       ALU only                           6
+#   multiplies                 multiply-add pipe only             6
+#   adds, high-word shifts,    either pipe, one op each           5 (fp32 word)
+#   and 4*hi + 1                                                  6 (16-bit word)
+#   funnel shifts              ALU, or two multiply-adds          3 (fp32), 2 (16-bit)
+# 20 operations per term when every flexible one runs on the ALU.
+TERM_OPS = {"f32": dict(alu_only=6, mul_only=6, flex=5, funnel=3),
+            "bf16": dict(alu_only=6, mul_only=6, flex=6, funnel=2)}
+ISSUE_LANES_PER_CLK_PER_SM = 128     # 4 schedulers x one 32-lane warp instruction per clock
+
+
+def integer_ceiling(words: dict, rates: dict) -> float:
+    """Elements per clock per SM at which the integer work of one element
+    (``words``: count of fp32 and 16-bit words digested per element) fits
+    the measured ALU and multiply-add lane rates and the issue width, with
+    the flexible operations split between the two pipes as well as
+    possible (a convex piecewise-linear minimum, scanned finely)."""
+    A0 = sum(n * (t["alu_only"] + t["flex"] + t["funnel"]) for k, n in words.items() for t in [TERM_OPS[k]])
+    F0 = sum(n * t["mul_only"] for k, n in words.items() for t in [TERM_OPS[k]])
+    n1 = sum(n * TERM_OPS[k]["flex"] for k, n in words.items())
+    nf = sum(n * TERM_OPS[k]["funnel"] for k, n in words.items())
+    ra = rates["alu"]["lane_ops_per_clk_per_sm"]
+    rf = rates["fma"]["lane_ops_per_clk_per_sm"]
+    ri = ISSUE_LANES_PER_CLK_PER_SM
+    best = None
+    steps = 4000
+    for i in range(steps + 1):
+        x = (n1 + nf) * i / steps                    # operations moved to the multiply-add pipe
+        extra = max(0.0, x - n1)                     # funnel shifts moved cost two multiply-adds each
+        t = max((A0 - x) / ra, (F0 + x + extra) / rf, (A0 + F0 + extra) / ri)
+        best = t if best is None or t < best else best
+    return 1.0 / best
+
 
 # What each synthetic workload stands for (synth/workloads.py).
 WORKLOAD_TEXT = {
@@ -64,6 +106,36 @@ WORKLOAD_TEXT = {
     "c4": "Mistral-7B rank shard 9 of 16, crossing tensor boundaries",
     "c5": "full Mistral-7B shard on one GPU",
 }
+
+
+def verify_roofline(rates, clk, n: int, v_ms: float, hbm_peak: float, launches: int, traffic):
+    """The verification pass (4 words per element: p', m', v' fp32 and w
+    bf16) against the lower of its integer ceiling, from the definition's
+    operation count and the measured lane rates at the sampled SM clock, and
+    its HBM ceiling (14 bytes per element at the measured copy bandwidth)."""
+    terms_per_s = 4 * n / (v_ms * 1e-3)
+    rec = {"kernel": "digest_kernel", "achieved": terms_per_s / 1e12, "unit": "T splitmix64 terms/s",
+           "launches": launches, "traffic": traffic, "algorithmic_bytes": VERIFY_BYTES * n,
+           "hbm_gbs": VERIFY_BYTES * n / (v_ms * 1e-3) / 1e9, "hbm_frac": VERIFY_BYTES * n / (v_ms * 1e-3) / 1e9 / hbm_peak}
+    hbm_terms = 4 * hbm_peak * 1e9 / VERIFY_BYTES
+    if rates is None:
+        rec.update(bound="hbm", peak=hbm_terms / 1e12, frac=terms_per_s / hbm_terms,
+                   peak_basis="integer rates not measured: HBM only")
+        return rec
+    sm_hz = (clk["sm_mhz"] if clk and clk.get("sm_mhz") else 2070.0) * 1e6
+    per_clk = integer_ceiling({"f32": 3, "bf16": 1}, rates)            # elements per clock per SM
+    int_terms = 4 * per_clk * rates["sms"] * sm_hz
+    bound, peak = ("alu", int_terms) if int_terms < hbm_terms else ("hbm", hbm_terms)
+    rec.update(bound=bound, peak=peak / 1e12, frac=terms_per_s / peak, integer_peak=int_terms / 1e12,
+               integer_frac=terms_per_s / int_terms, hbm_peak_terms=hbm_terms / 1e12,
+               measured_lane_ops_per_clk_per_sm={k: rates[k]["lane_ops_per_clk_per_sm"] for k in ("alu", "fma", "both")},
+               sm_mhz=sm_hz / 1e6,
+               peak_basis="splitmix64 as defined, 20 32-bit operations per term (6 xors on the ALU, 6 multiply-adds, "
+                          "the adds and shifts on either pipe, a funnel shift costing two multiply-adds off the "
+                          "ALU), split as well as possible over the ALU and multiply-add lane rates measured by "
+                          "register-only probes (libapc_probe.so) and 128 issue lanes per clock per SM, at the "
+                          "sampled SM clock; against 14 B/element at the measured HBM bandwidth")
+    return rec
 
 
 def measured_peak():
@@ -97,6 +169,33 @@ def kernel_source_hash(kernel: str) -> str:
         code = " ".join(code.split())
         h.update(name.encode() + code.encode())
     return h.hexdigest()[:16]
+
+
+def profiled_field(kernel: str, field: str):
+    """A figure of ``kernel`` from the committed ncu summary, if it was taken
+    on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[kernel]
+    except (OSError, KeyError, ValueError):
+        return None
+    src = KERNEL_SOURCES.get(kernel.replace("_bf16", ""))
+    if src is None or rec.get("source_hash") != kernel_source_hash(kernel.replace("_bf16", "")):
+        return None
+    return rec.get(field)
+
+
+def issue_ceiling(kernel: str, n: int, ms: float, sms: int, clk) -> dict | None:
+    """The instruction-issue ceiling of a commit launch: its ncu instruction
+    count per element x elements over 128 issue lanes per clock per SM at the
+    sampled SM clock."""
+    ipe = profiled_field(kernel, "inst_per_element")
+    if ipe is None:
+        return None
+    sm_hz = (clk["sm_mhz"] if clk and clk.get("sm_mhz") else 2070.0) * 1e6
+    t = ipe * n / (sms * ISSUE_LANES_PER_CLK_PER_SM * sm_hz)
+    return {"inst_per_element": ipe, "ceiling_ms": t * 1e3, "frac": t * 1e3 / ms, "sm_mhz": sm_hz / 1e6}
 
 
 def profiled_traffic(kernel: str, workload: str):
@@ -412,6 +511,13 @@ def run_gpu(args):
     # stream; later steps update the state in place.
     first_digests = apc.digests_to_host(apc.commit_step(tab, step_t, HP, stream=s, out=out_c))
 
+    def grid_limit(n):
+        # APC_GRID_LIMIT is read by every library call (include/apc.h)
+        if n:
+            os.environ["APC_GRID_LIMIT"] = str(n)
+        else:
+            os.environ.pop("APC_GRID_LIMIT", None)
+
     def one_step(ev=None):
         if ev is not None:
             ev[0].record(stream)
@@ -422,23 +528,70 @@ def run_gpu(args):
         if ev is not None:
             ev[2].record(stream)
 
+    if args.schedule == "pipelined":
+        # The table cut into groups; the verification of group g runs on a
+        # second stream once group g's commit is done, beside the commits of
+        # the later groups.  ev[1] marks the end of the last commit, ev[2] the
+        # end of the last verification.
+        pgroups = group_pieces([pc.n for pc in w.pieces], args.groups)
+        ptab = [apc.prepare_table([entries[k] for k in idx]) for idx in pgroups]
+        pvtab = [apc.prepare_buffers([vbufs[4 * k + j] for k in idx for j in range(4)]) for idx in pgroups]
+        pout = torch.empty(len(pgroups), 8, dtype=torch.int64, device=dev)
+        vstream = torch.cuda.Stream(device=dev)
+        pdone = [torch.cuda.Event() for _ in pgroups]
+
+        def one_step(ev=None):  # noqa: F811 (the pipelined schedule replaces the sequential one)
+            if ev is not None:
+                ev[0].record(stream)
+            for gi in range(len(pgroups)):
+                grid_limit(args.commit_grid)
+                apc.commit_step(ptab[gi], step_t, HP, stream=s, out=pout[gi, :4])
+                pdone[gi].record(stream)
+                vstream.wait_event(pdone[gi])
+                grid_limit(args.verify_grid)
+                apc.digest(pvtab[gi], 4, stream=vstream.cuda_stream, out=pout[gi, 4:])
+            grid_limit(0)
+            if ev is not None:
+                ev[1].record(stream)
+            stream.wait_stream(vstream)
+            out_c.copy_(pout[:, :4].sum(0))
+            out_v.copy_(pout[:, 4:].sum(0))
+            if ev is not None:
+                ev[2].record(stream)
+
     for _ in range(args.warmup):
         one_step()
     torch.cuda.synchronize()
 
     K = args.steps
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    # A step whose bytes fit in L2 would find its inputs there: write a
+    # buffer twice the L2's size between timed steps, outside their events.
+    flush = (torch.empty(2 * L2_BYTES // 4, dtype=torch.int32, device=dev)
+             if (COMMIT_BYTES + VERIFY_BYTES) * N <= 4 * L2_BYTES else None)
     clocks = ClockSampler(local) if not args.no_clocks else None
     barrier(dist)
     torch.cuda.synchronize()
     for k in range(K):
+        if flush is not None:
+            flush.fill_(k)
         one_step(evs[k])
     torch.cuda.synchronize()
     barrier(dist)
     clk = clocks.stop() if clocks else None
+    rates = None
+    if rank == 0:
+        try:
+            from paper_2609_18178_gb300 import peak as apc_peak
+            rates = apc_peak.int_rates()
+        except (OSError, RuntimeError, subprocess.CalledProcessError) as ex:
+            print("note: integer-rate probe unavailable (%s); verify roofline against HBM only" % ex, file=sys.stderr)
     commit_ms = [evs[k][0].elapsed_time(evs[k][1]) for k in range(K)]
     verify_ms = [evs[k][1].elapsed_time(evs[k][2]) for k in range(K)]
-    total_ms = evs[0][0].elapsed_time(evs[K - 1][2])
+    if flush is None:
+        total_ms = evs[0][0].elapsed_time(evs[K - 1][2])
+    else:   # per-step events only: the flushes between them are not timed
+        total_ms = sum(evs[k][0].elapsed_time(evs[k][2]) for k in range(K))
     total_ms = max_over_ranks(dist, total_ms)
     ms_per_step = total_ms / K
     digests_c = apc.digests_to_host(out_c)
@@ -593,6 +746,8 @@ def run_gpu(args):
                 ms.append(a0.elapsed_time(a1))
             return statistics.median(ms)
 
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        sm_hz = (clk["sm_mhz"] if clk and clk.get("sm_mhz") else 2070.0) * 1e6
         nz_before = apc.digests_to_host(apc.count_nonzero(gbufs, 1, stream=s, out=out_n))[0]
         guard_ms = timed(lambda: apc.count_nonzero(gbufs, 1, stream=s, out=out_n), max(3, K))
         zero_ms = timed(lambda: apc.commit_step(tab, step_t, HP, stream=s, out=out_c, zero_grad=True), max(3, K))
@@ -626,7 +781,14 @@ def run_gpu(args):
                                                     % (N3, len(w3.pieces)), "ms": f3_ms, "gbs": 14 * N3 / (f3_ms * 1e-3) / 1e9,
                                         "frac": 14 * N3 / (f3_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 14,
                                         "verify_ms": f3v_ms, "verify_gbs": 6 * N3 / (f3v_ms * 1e-3) / 1e9,
-                                        "verify_matches_commit": f3_ok},
+                                        "verify_frac": 6 * N3 / (f3v_ms * 1e-3) / 1e9 / peak_n,
+                                        "verify_matches_commit": f3_ok,
+                                        "issue": issue_ceiling("commit_kernel_bf16", N3, f3_ms, sms, clk),
+                                        "verify_integer": (None if rates is None else
+                                                           {"ceiling_ms": 1e3 * N3 / (integer_ceiling({"bf16": 3}, rates)
+                                                                                     * rates["sms"] * sm_hz),
+                                                            "frac": 1e3 * N3 / (integer_ceiling({"bf16": 3}, rates)
+                                                                                * rates["sms"] * sm_hz) / f3v_ms})},
                "f1_commit_zero_grad": {"ms": zero_ms, "gbs": 30 * N / (zero_ms * 1e-3) / 1e9,
                                        "frac": 30 * N / (zero_ms * 1e-3) / 1e9 / peak_n, "bytes_per_element": 30},
                "f1_guard_count_nonzero": {"ms": guard_ms, "gbs": 2 * N / (guard_ms * 1e-3) / 1e9,
@@ -652,6 +814,8 @@ def run_gpu(args):
     peak, peak_kind = measured_peak()
     n_commit_launches = max(1, (len(entries) + 439) // 440)
     n_digest_launches = max(1, (len(vbufs) + 999) // 1000)
+    if args.schedule == "pipelined":
+        n_commit_launches = n_digest_launches = len(group_pieces([pc.n for pc in w.pieces], args.groups))
     c_ms = statistics.median(commit_ms)
     v_ms = statistics.median(verify_ms)
     c_avg = sum(commit_ms) / K
@@ -678,9 +842,10 @@ def run_gpu(args):
                    "parallelism": ("%d ranks x one contiguous range of the flat model each (no data-path "
                                    "collective)" % world if args.split == "model" else
                                    "%d ranks x one full-size shard each (no data-path collective)" % world),
-                   "l2": ("inputs larger than L2 (%.1f GB resident state)" % (16 * N / 1e9)
-                          if COMMIT_BYTES * N > L2_BYTES else
-                          "inputs smaller than L2 (%.3f GB per step): timings include L2 hits" % (COMMIT_BYTES * N / 1e9))},
+                   "l2": ("inputs larger than L2 (%.1f GB resident state)" % (16 * N / 1e9) if flush is None else
+                          "L2 flushed between timed steps (a %d MB write outside the step's events): the step's "
+                          "%.3f GB would otherwise fit in L2" % (2 * L2_BYTES >> 20,
+                                                                  (COMMIT_BYTES + VERIFY_BYTES) * N / 1e9))},
         "hbm_gbs_step": (COMMIT_BYTES + VERIFY_BYTES) * N / (ms_per_step * 1e-3) / 1e9,
         "commit_ms": c_ms,
         "verify_ms": v_ms,
@@ -688,19 +853,25 @@ def run_gpu(args):
         "verify_gbs": VERIFY_BYTES * N / (v_ms * 1e-3) / 1e9,
         "commit_elements_per_s": N / (c_ms * 1e-3),
         "frac_of_spec_8tbs": achieved / 8000.0,
-        "roofline": {"bound": "hbm", "kernel": "commit_kernel", "achieved": achieved, "peak": peak,
+        "roofline": None if args.schedule == "pipelined" else {"bound": "hbm", "kernel": "commit_kernel",
+                     "achieved": achieved, "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                     "frac_of_spec_8tbs": achieved / 8000.0,
                      "traffic": profiled_traffic("commit_kernel", w.name),
-                     "algorithmic_bytes_per_launch": COMMIT_BYTES * N},
-        "roofline_verify": {"bound": "alu", "kernel": "digest_kernel", "achieved": 4 * N / (v_avg * 1e-3) / 1e12,
-                            "peak": ALU_LANE_OPS_PER_S / VERIFY_ALU_INSTRUCTIONS_PER_TERM / 1e12,
-                            "unit": "T splitmix64 terms/s",
-                            "frac": 4 * N / (v_avg * 1e-3) / (ALU_LANE_OPS_PER_S / VERIFY_ALU_INSTRUCTIONS_PER_TERM),
-                            "peak_basis": "152 SMs x 64 integer-ALU lanes x 2.07 GHz over %.1f ALU instructions "
-                                          "per term" % VERIFY_ALU_INSTRUCTIONS_PER_TERM,
-                            "launches": n_digest_launches,
-                            "traffic": profiled_traffic("digest_kernel", w.name),
-                            "algorithmic_bytes": VERIFY_BYTES * N},
+                     "traffic_note": ("ncu DRAM bytes of the 152M-element c3 launch scaled by elements: a lower "
+                                      "bound, since writes still in L2 when that launch ended are not counted"),
+                     "algorithmic_bytes_per_launch": COMMIT_BYTES * N,
+                     "issue": issue_ceiling("commit_kernel", N, c_avg, torch.cuda.get_device_properties(dev)
+                                            .multi_processor_count, clk)},
+        "roofline_verify": None if args.schedule == "pipelined" else verify_roofline(
+            rates, clk, N, v_avg, peak, n_digest_launches, profiled_traffic("digest_kernel", w.name)),
+        "schedule": ({"kind": "sequential"} if args.schedule == "sequential" else
+                     {"kind": "pipelined", "groups": args.groups, "commit_grid": args.commit_grid or "default",
+                      "verify_grid": args.verify_grid or "default", "commit_span_ms": c_ms,
+                      "verify_tail_ms": v_ms,
+                      "note": "commit and verification kernels overlap: commit_ms is the span of the commit "
+                              "stream, verify_ms the verification tail after it, and the kernel rooflines are "
+                              "those of the sequential schedule, not measured here"}),
         "gpu_launches": K * (n_commit_launches + n_digest_launches),
         "gpu_launches_note": "per timed step: %d commit_kernel + %d digest_kernel launches (%d tensors, %d buffers; "
                              "up to 440 tensors and 1000 buffers per launch)"
@@ -912,6 +1083,14 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["c1", "c2", "c3", "c4", "c5"], default="c5")
+    ap.add_argument("--schedule", choices=["sequential", "pipelined"], default="sequential",
+                    help="sequential: commit, then verify, on one stream; pipelined: the table in --groups groups, "
+                         "each group's verification on a second stream beside the next groups' commits")
+    ap.add_argument("--groups", type=int, default=12, help="groups of the pipelined schedule")
+    ap.add_argument("--commit-grid", type=int, default=0,
+                    help="pipelined schedule: CTAs of each commit launch (0: the library's persistent grid)")
+    ap.add_argument("--verify-grid", type=int, default=0,
+                    help="pipelined schedule: CTAs of each verification launch (0: the library's grid)")
     ap.add_argument("--split", choices=["copy", "model"], default="copy",
                     help="multi-GPU: every rank a full-size copy of the workload (copy, weak scaling) or rank r "
                          "the contiguous range r of the one model's flat parameters (model, strong scaling)")

@@ -128,6 +128,7 @@ struct F32State {
   static constexpr int kConsumerWarps = kCommitConsumerWarps;
   static constexpr int kConsumers = 32 * kConsumerWarps;
   static constexpr int kThreads = kConsumers + 32;  // + the producer warp
+  static constexpr int kBoundThreads = kThreads > APC_COMMIT_BOUND_THREADS ? kThreads : APC_COMMIT_BOUND_THREADS;
   static constexpr int kGroups = kCommitGroups;
   static constexpr uint64_t kTile = kCommitTile;
   struct Regs {
@@ -207,6 +208,7 @@ struct BF16State {
   static constexpr int kConsumerWarps = kCommitConsumerWarpsBF16;
   static constexpr int kConsumers = 32 * kConsumerWarps;
   static constexpr int kThreads = kConsumers + 32;
+  static constexpr int kBoundThreads = kThreads;
   static constexpr int kGroups = kCommitGroupsBF16;
   static constexpr uint64_t kTile = kCommitTileBF16;
   struct Regs {
@@ -312,7 +314,7 @@ __device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint
 }
 
 template <class L, int MAXE, bool ZERO>
-__global__ void __launch_bounds__(L::kThreads, kCommitBlocksPerSm)
+__global__ void __launch_bounds__(L::kBoundThreads, kCommitBlocksPerSm)
     commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan, unsigned long long *out) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ __align__(8) uint64_t full[kCommitStages];
@@ -476,6 +478,11 @@ int ensure_smem_attribute() {
   e = cudaFuncSetAttribute(commit_kernel<L, MAXE, ZERO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem_bytes<L>());
   if (e != cudaSuccess) return (int)e;
+  if (APC_SMEM_CARVEOUT >= 0) {
+    e = cudaFuncSetAttribute(commit_kernel<L, MAXE, ZERO>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             APC_SMEM_CARVEOUT);
+    if (e != cudaSuccess) return (int)e;
+  }
   if (bit) done_mask.fetch_or(bit, std::memory_order_acq_rel);
   return 0;
 }

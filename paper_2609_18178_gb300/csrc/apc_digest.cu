@@ -142,6 +142,7 @@ __device__ __forceinline__ void last_tile_ok(uint64_t base, uint64_t vec_end, bo
 // slot are contiguous.
 constexpr int kStageSlots = 2 * kDigestUnroll;                       // 16-byte words per thread per stage
 constexpr uint32_t kStageBytes = 2u * kStageSlots * kThreads * 16u;  // two stages: 73,728 bytes
+constexpr uint32_t kLaunchSmem = kStageBytes + APC_DIGEST_EXTRA_SMEM;
 
 __device__ __forceinline__ void cp16(uint32_t dst, const void *src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -166,7 +167,7 @@ __device__ __forceinline__ uint32_t word_at(const DigestEntry &E, uint64_t i) {
 // compiler use 80 registers: without per-vector checks a full tile's 24 terms
 // form one block that it schedules for more overlap than 64 registers hold.
 template <int MAXE>
-__global__ void __launch_bounds__(kThreads, 2) digest_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
+__global__ void __launch_bounds__(kThreads, APC_DIGEST_MIN_BLOCKS) digest_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
                                                           unsigned long long *out) {
   __shared__ unsigned long long s_acc[APC_MAX_SLOTS];
   extern __shared__ __align__(16) uint4 stg[];
@@ -298,8 +299,12 @@ int ensure_stage_attribute() {
   if (e != cudaSuccess) return (int)e;
   const uint64_t bit = dev < 64 ? (1ull << dev) : 0;
   if (bit && (done_mask.load(std::memory_order_acquire) & bit)) return 0;
-  e = cudaFuncSetAttribute(digest_kernel<MAXE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStageBytes);
+  e = cudaFuncSetAttribute(digest_kernel<MAXE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kLaunchSmem);
   if (e != cudaSuccess) return (int)e;
+  if (APC_SMEM_CARVEOUT >= 0) {
+    e = cudaFuncSetAttribute(digest_kernel<MAXE>, cudaFuncAttributePreferredSharedMemoryCarveout, APC_SMEM_CARVEOUT);
+    if (e != cudaSuccess) return (int)e;
+  }
   if (bit) done_mask.fetch_or(bit, std::memory_order_acq_rel);
   return 0;
 }
@@ -308,7 +313,7 @@ template <int MAXE>
 int launch_t(const DigestPlan<MAXE> &plan, unsigned grid, void *stream, unsigned long long *out) {
   int e = ensure_stage_attribute<MAXE>();
   if (e) return e;
-  digest_kernel<MAXE><<<grid, kThreads, kStageBytes, (cudaStream_t)stream>>>(plan, out);
+  digest_kernel<MAXE><<<grid, kThreads, kLaunchSmem, (cudaStream_t)stream>>>(plan, out);
   return (int)cudaGetLastError();
 }
 
@@ -316,7 +321,7 @@ template <int MAXE>
 int blocks_t(int *out) {
   int e = ensure_stage_attribute<MAXE>();
   if (e) return e;
-  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<MAXE>, kThreads, kStageBytes);
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, digest_kernel<MAXE>, kThreads, kLaunchSmem);
 }
 
 }  // namespace

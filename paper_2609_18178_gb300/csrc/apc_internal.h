@@ -57,6 +57,19 @@ constexpr uint64_t kCommitTile = (uint64_t)kCommitConsumerWarps * 32 * 4 * kComm
 constexpr uint64_t kCommitTileBF16 = (uint64_t)kCommitConsumerWarpsBF16 * 32 * 4 * kCommitGroupsBF16;  // 10,368 elements
 constexpr int kCommitStages = APC_COMMIT_STAGES;
 constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
+// Register budget of the fp32-state commit kernel: its launch bound is
+// max(block size, APC_COMMIT_BOUND_THREADS) threads, so a build with fewer
+// consumer warps can keep the default 96 registers per thread (and leave the
+// rest of the SM to a co-resident kernel) instead of growing into them.
+#ifndef APC_COMMIT_BOUND_THREADS
+#define APC_COMMIT_BOUND_THREADS 0
+#endif
+// Shared-memory carveout preference (percent of the unified L1/shared
+// capacity) given to the commit and digest kernels; -1 leaves the driver's
+// default.  100 lets two different kernels' CTAs share an SM.
+#ifndef APC_SMEM_CARVEOUT
+#define APC_SMEM_CARVEOUT -1
+#endif
 // A stage holds one tile of p, m, v and g: 14 bytes per element for fp32
 // state (133 KB per CTA at the defaults), 8 for bf16 state (162 KB).
 
@@ -117,6 +130,16 @@ static_assert(sizeof(CommitPlan<kCommitLarge>) <= 32764, "kernel parameter limit
 constexpr int kThreads = APC_DIGEST_THREADS;     // threads per CTA of the digest kernel
 constexpr int kDigestUnroll = APC_DIGEST_UNROLL; // thread-vectors per thread per tile
 constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 9,216 elements
+// Minimum resident CTAs per SM the digest kernel is compiled for (its
+// register cap: 65,536 / (threads x this)), and extra dynamic shared memory
+// per CTA beyond its stages (0 by default; a larger CTA footprint keeps two
+// digest CTAs off one SM when another kernel is to share it).
+#ifndef APC_DIGEST_MIN_BLOCKS
+#define APC_DIGEST_MIN_BLOCKS 2
+#endif
+#ifndef APC_DIGEST_EXTRA_SMEM
+#define APC_DIGEST_EXTRA_SMEM 0
+#endif
 
 // One buffer of the digest kernel (32 bytes).
 //   head: scalar elements before the first 16-byte boundary (<= 7); then

@@ -1,0 +1,78 @@
+// Register-only throughput probes of the SM's integer pipes, the measured
+// denominators of the verification pass's roofline.  Not part of the hot
+// path: libapc_probe.so is a separate library that the benchmark loads.
+//
+// Every thread runs `iters` steps over kChains independent chains held in
+// registers; no memory is touched between the two clock reads.  A step is:
+//   kind 0 (ALU pipe): a 32-bit funnel shift and an xor       2 lane-ops
+//   kind 1 (multiply-add pipe): two 32-bit multiply-adds      2 lane-ops
+//   kind 2 (both): the two ALU operations and the two
+//          multiply-adds of kinds 0 and 1, interleaved          4 lane-ops
+// The operands of each operation come from the previous step, so the
+// compiler can neither fold nor hoist them.  Thread 0 of every CTA records
+// the SM clocks its CTA spent in the loop; all CTAs of the grid run at once
+// (grid = SMs x 2 CTAs of 512 threads), so lane-ops / (cycles x SMs) is the
+// SM's rate per clock, independent of the clock frequency.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#define APC_PROBE_EXPORT extern "C" __attribute__((visibility("default")))
+
+namespace {
+
+constexpr int kChains = 8;
+constexpr int kProbeThreads = 512;
+
+template <int KIND>
+__global__ void __launch_bounds__(kProbeThreads, 2)
+    int_rate_kernel(uint32_t iters, uint32_t seed, uint32_t *sink, unsigned long long *cycles) {
+  uint32_t a[kChains], b[kChains];
+#pragma unroll
+  for (int k = 0; k < kChains; ++k) {
+    a[k] = seed ^ (threadIdx.x * kChains + k);
+    b[k] = a[k] * 0x9E3779B9u + 0x7F4A7C15u;
+  }
+  __syncthreads();
+  const long long t0 = clock64();
+  for (uint32_t i = 0; i < iters; ++i) {
+#pragma unroll
+    for (int k = 0; k < kChains; ++k) {
+      if (KIND != 1) {
+        uint32_t t;
+        asm volatile("shf.r.wrap.b32 %0, %1, %2, 7;" : "=r"(t) : "r"(a[k]), "r"(b[k]));
+        asm volatile("xor.b32 %0, %0, %1;" : "+r"(a[k]) : "r"(t));
+      }
+      if (KIND != 0) {
+        asm volatile("mad.lo.u32 %0, %0, %1, 0x7F4A7C15;" : "+r"(b[k]) : "r"(a[k]));
+        asm volatile("mad.lo.u32 %0, %0, %1, 0x1CE4E5B9;" : "+r"(a[k]) : "r"(b[k]));
+      }
+    }
+  }
+  __syncthreads();
+  const long long t1 = clock64();
+  uint32_t x = 0;
+#pragma unroll
+  for (int k = 0; k < kChains; ++k) x ^= a[k] + b[k];
+  sink[blockIdx.x * blockDim.x + threadIdx.x] = x;
+  if (threadIdx.x == 0) cycles[blockIdx.x] = (unsigned long long)(t1 - t0);
+}
+
+}  // namespace
+
+// Launch one probe on `stream`: kind 0, 1 or 2 (see above), `iters` steps,
+// `grid` CTAs of 512 threads.  sink: device, grid x 512 uint32 (written);
+// cycles: device, grid uint64 (written: the SM clocks of each CTA's loop).
+// Returns 0 or a cudaError_t value.  Lane-ops per CTA:
+// 512 x iters x 8 x (2, 2 or 4).
+APC_PROBE_EXPORT int apc_probe_int_rate(int kind, uint32_t iters, uint32_t grid, uint32_t *sink,
+                                        unsigned long long *cycles, void *stream) {
+  if (kind < 0 || kind > 2 || grid == 0 || !sink || !cycles) return (int)cudaErrorInvalidValue;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (kind == 0) int_rate_kernel<0><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, cycles);
+  else if (kind == 1) int_rate_kernel<1><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, cycles);
+  else int_rate_kernel<2><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, cycles);
+  return (int)cudaGetLastError();
+}
+
+APC_PROBE_EXPORT int apc_probe_threads(void) { return kProbeThreads; }
+APC_PROBE_EXPORT int apc_probe_chains(void) { return kChains; }

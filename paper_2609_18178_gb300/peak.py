@@ -1,0 +1,70 @@
+"""Measured integer-pipe rates of the current GPU, from the register-only
+probes of ``libapc_probe.so`` (csrc/apc_probe.cu).  The benchmark divides
+the verification pass's work, counted from the splitmix64 definition, by
+these rates to form its roofline; nothing in the hot path uses them.
+
+``int_rates()`` returns, for each probe kind, the SM's lane-operations per
+clock (from the kernel's own clock64 readings, independent of the clock
+frequency) and lane-operations per second (from CUDA events on the launching
+stream, at whatever clock the GPU ran).
+"""
+from __future__ import annotations
+
+import ctypes
+import statistics
+
+from . import _build
+
+KINDS = {"alu": 0, "fma": 1, "both": 2}
+OPS_PER_STEP = {"alu": 2, "fma": 2, "both": 4}
+
+_lib = None
+
+
+def library():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(_build.build_probe())
+        lib.apc_probe_int_rate.argtypes = [ctypes.c_int, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_void_p,
+                                           ctypes.c_void_p, ctypes.c_void_p]
+        lib.apc_probe_int_rate.restype = ctypes.c_int
+        lib.apc_probe_threads.restype = ctypes.c_int
+        lib.apc_probe_chains.restype = ctypes.c_int
+        _lib = lib
+    return _lib
+
+
+def int_rates(iters: int = 8192, reps: int = 5) -> dict:
+    """Lane-op rates of the ALU pipe ("alu": funnel shifts and xors), the
+    multiply-add pipe ("fma": 32-bit multiply-adds) and both together
+    ("both": equal numbers, the issue-limited mix), on a grid of two
+    512-thread CTAs per SM; median of ``reps`` launches after one warm-up."""
+    import torch
+    lib = library()
+    dev = torch.cuda.current_device()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    grid = 2 * sms
+    threads, chains = lib.apc_probe_threads(), lib.apc_probe_chains()
+    sink = torch.empty(grid * threads, dtype=torch.int32, device="cuda")
+    cycles = torch.empty(grid, dtype=torch.int64, device="cuda")
+    stream = torch.cuda.current_stream()
+    out = {"sms": sms, "grid": grid, "threads": threads, "iters": iters}
+    for name, kind in KINDS.items():
+        per_cta = threads * iters * chains * OPS_PER_STEP[name]
+        clk, sec = [], []
+        for r in range(reps + 1):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            rc = lib.apc_probe_int_rate(kind, iters, grid, ctypes.c_void_p(sink.data_ptr()),
+                                        ctypes.c_void_p(cycles.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
+            if rc:
+                raise RuntimeError("integer-rate probe launch failed (cudaError %d)" % rc)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if r == 0:
+                continue
+            cyc = statistics.median(int(x) for x in cycles.cpu().tolist())
+            clk.append(2 * per_cta / cyc)                     # two CTAs share each SM for the whole loop
+            sec.append(grid * per_cta / (e0.elapsed_time(e1) * 1e-3))
+        out[name] = {"lane_ops_per_clk_per_sm": statistics.median(clk), "lane_ops_per_s": statistics.median(sec)}
+    return out
