@@ -10,9 +10,10 @@
 //          multiply-adds of kinds 0 and 1, interleaved          4 lane-ops
 // The operands of each operation come from the previous step, so the
 // compiler can neither fold nor hoist them.  Thread 0 of every CTA records
-// the SM clocks its CTA spent in the loop; all CTAs of the grid run at once
-// (grid = SMs x 2 CTAs of 512 threads), so lane-ops / (cycles x SMs) is the
-// SM's rate per clock, independent of the clock frequency.
+// its SM's id and the SM clock counter when the CTA's loop starts and ends;
+// per SM, the lane-ops of all CTAs it ran over the span from the first start
+// to the last end is the SM's rate per clock, independent of the clock
+// frequency and of how the CTAs were placed.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -21,11 +22,11 @@
 namespace {
 
 constexpr int kChains = 8;
-constexpr int kProbeThreads = 512;
+constexpr int kProbeThreads = 1024;
 
 template <int KIND>
-__global__ void __launch_bounds__(kProbeThreads, 2)
-    int_rate_kernel(uint32_t iters, uint32_t seed, uint32_t *sink, unsigned long long *cycles) {
+__global__ void __launch_bounds__(kProbeThreads)
+    int_rate_kernel(uint32_t iters, uint32_t seed, uint32_t *sink, unsigned long long *clocks) {
   uint32_t a[kChains], b[kChains];
 #pragma unroll
   for (int k = 0; k < kChains; ++k) {
@@ -54,23 +55,29 @@ __global__ void __launch_bounds__(kProbeThreads, 2)
 #pragma unroll
   for (int k = 0; k < kChains; ++k) x ^= a[k] + b[k];
   sink[blockIdx.x * blockDim.x + threadIdx.x] = x;
-  if (threadIdx.x == 0) cycles[blockIdx.x] = (unsigned long long)(t1 - t0);
+  if (threadIdx.x == 0) {
+    uint32_t sm;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
+    clocks[3 * blockIdx.x] = sm;
+    clocks[3 * blockIdx.x + 1] = (unsigned long long)t0;
+    clocks[3 * blockIdx.x + 2] = (unsigned long long)t1;
+  }
 }
 
 }  // namespace
 
 // Launch one probe on `stream`: kind 0, 1 or 2 (see above), `iters` steps,
-// `grid` CTAs of 512 threads.  sink: device, grid x 512 uint32 (written);
-// cycles: device, grid uint64 (written: the SM clocks of each CTA's loop).
-// Returns 0 or a cudaError_t value.  Lane-ops per CTA:
-// 512 x iters x 8 x (2, 2 or 4).
+// `grid` CTAs of 1024 threads.  sink: device, grid x 1024 uint32 (written);
+// clocks: device, 3 x grid uint64 (written: per CTA its SM id and the SM
+// clock counter at the start and the end of its loop).  Returns 0 or a
+// cudaError_t value.  Lane-ops per CTA: 1024 x iters x 8 x (2, 2 or 4).
 APC_PROBE_EXPORT int apc_probe_int_rate(int kind, uint32_t iters, uint32_t grid, uint32_t *sink,
-                                        unsigned long long *cycles, void *stream) {
-  if (kind < 0 || kind > 2 || grid == 0 || !sink || !cycles) return (int)cudaErrorInvalidValue;
+                                        unsigned long long *clocks, void *stream) {
+  if (kind < 0 || kind > 2 || grid == 0 || !sink || !clocks) return (int)cudaErrorInvalidValue;
   cudaStream_t s = (cudaStream_t)stream;
-  if (kind == 0) int_rate_kernel<0><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, cycles);
-  else if (kind == 1) int_rate_kernel<1><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, cycles);
-  else int_rate_kernel<2><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, cycles);
+  if (kind == 0) int_rate_kernel<0><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
+  else if (kind == 1) int_rate_kernel<1><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
+  else int_rate_kernel<2><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
   return (int)cudaGetLastError();
 }
 

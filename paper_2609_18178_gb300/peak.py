@@ -37,16 +37,18 @@ def library():
 def int_rates(iters: int = 8192, reps: int = 5) -> dict:
     """Lane-op rates of the ALU pipe ("alu": funnel shifts and xors), the
     multiply-add pipe ("fma": 32-bit multiply-adds) and both together
-    ("both": equal numbers, the issue-limited mix), on a grid of two
-    512-thread CTAs per SM; median of ``reps`` launches after one warm-up."""
+    ("both": equal numbers, the issue-limited mix), on a grid of one
+    1024-thread CTA per SM; median of ``reps`` launches after one warm-up.
+    Per clock: each SM's lane-ops over the span of its SM clock counter from
+    its first CTA's start to its last CTA's end, median over the SMs."""
     import torch
     lib = library()
     dev = torch.cuda.current_device()
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    grid = 2 * sms
+    grid = sms
     threads, chains = lib.apc_probe_threads(), lib.apc_probe_chains()
     sink = torch.empty(grid * threads, dtype=torch.int32, device="cuda")
-    cycles = torch.empty(grid, dtype=torch.int64, device="cuda")
+    clocks = torch.empty(3 * grid, dtype=torch.int64, device="cuda")
     stream = torch.cuda.current_stream()
     out = {"sms": sms, "grid": grid, "threads": threads, "iters": iters}
     for name, kind in KINDS.items():
@@ -56,15 +58,20 @@ def int_rates(iters: int = 8192, reps: int = 5) -> dict:
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             rc = lib.apc_probe_int_rate(kind, iters, grid, ctypes.c_void_p(sink.data_ptr()),
-                                        ctypes.c_void_p(cycles.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
+                                        ctypes.c_void_p(clocks.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
             if rc:
                 raise RuntimeError("integer-rate probe launch failed (cudaError %d)" % rc)
             e1.record(stream)
             torch.cuda.synchronize()
             if r == 0:
                 continue
-            cyc = statistics.median(int(x) for x in cycles.cpu().tolist())
-            clk.append(2 * per_cta / cyc)                     # two CTAs share each SM for the whole loop
+            c = clocks.cpu().tolist()
+            span = {}
+            for b in range(grid):
+                sm, t0, t1 = c[3 * b], c[3 * b + 1], c[3 * b + 2]
+                lo, hi, n = span.get(sm, (t0, t1, 0))
+                span[sm] = (min(lo, t0), max(hi, t1), n + 1)
+            clk.append(statistics.median(n * per_cta / (hi - lo) for lo, hi, n in span.values()))
             sec.append(grid * per_cta / (e0.elapsed_time(e1) * 1e-3))
         out[name] = {"lane_ops_per_clk_per_sm": statistics.median(clk), "lane_ops_per_s": statistics.median(sec)}
     return out

@@ -49,7 +49,7 @@ def run_ranks(world: int) -> dict:
     for p, (out, err) in zip(procs, outs):
         assert p.returncode == 0, err[-3000:]
     lines = [x for x in outs[0][0].splitlines() if x.startswith("{")]
-    assert len(lines) == 1 and all(not o.strip() for o, _ in outs[1:])   # rank 0 alone prints
+    assert len(lines) == 1 and not any(x.startswith("{") for o, _ in outs[1:] for x in o.splitlines())  # rank 0 alone prints the line
     return json.loads(lines[0])
 
 

@@ -98,3 +98,13 @@ def test_fill_is_position_pure_and_thread_invariant():
         idx = np.array([(1 << 32) - 1000 + j for j in (0, 1, 999, 1000, 1001, n - 1)], dtype=np.uint64)
         c = synth.fill_at(kind, idx, step=3)
         assert np.array_equal(c.view(np.uint8), a[idx - idx[0]].view(np.uint8))
+
+
+def test_lane_block_fill_equals_scalar_values():
+    """The host fill's 16-lane blocks give the scalar recipe's bits for
+    every kind, on ragged ranges (block remainders) across 2^32."""
+    for kind in (synth.P, synth.M, synth.V, synth.G, synth.P16, synth.M16, synth.V16):
+        for goff, n in ((0, 1000), ((1 << 32) - 37, 5003), (12_345_678_901, 777), (5, 15), (7, 16), (9, 17)):
+            a = synth.fill(kind, n, goff, step=7, nthreads=3)
+            b = synth.fill_at(kind, np.arange(goff, goff + n, dtype=np.uint64), step=7)
+            assert np.array_equal(a.view(np.uint8), b.view(np.uint8)), (kind, goff, n)
