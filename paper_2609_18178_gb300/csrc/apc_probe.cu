@@ -8,6 +8,9 @@
 //   kind 1 (multiply-add pipe): two 32-bit multiply-adds      2 lane-ops
 //   kind 2 (both): the two ALU operations and the two
 //          multiply-adds of kinds 0 and 1, interleaved          4 lane-ops
+//   kind 3 (high multiply): two 32-bit high multiply-adds     2 lane-ops
+//   kind 4 (wide multiply): two 32 x 32 -> 64-bit
+//          multiply-adds                                      2 lane-ops
 // The operands of each operation come from the previous step, so the
 // compiler can neither fold nor hoist them.  Thread 0 of every CTA records
 // its SM's id and the SM clock counter when the CTA's loop starts and ends;
@@ -38,14 +41,24 @@ __global__ void __launch_bounds__(kProbeThreads)
   for (uint32_t i = 0; i < iters; ++i) {
 #pragma unroll
     for (int k = 0; k < kChains; ++k) {
-      if (KIND != 1) {
+      if (KIND == 0 || KIND == 2) {
         uint32_t t;
         asm volatile("shf.r.wrap.b32 %0, %1, %2, 7;" : "=r"(t) : "r"(a[k]), "r"(b[k]));
         asm volatile("xor.b32 %0, %0, %1;" : "+r"(a[k]) : "r"(t));
       }
-      if (KIND != 0) {
+      if (KIND == 1 || KIND == 2) {
         asm volatile("mad.lo.u32 %0, %0, %1, 0x7F4A7C15;" : "+r"(b[k]) : "r"(a[k]));
         asm volatile("mad.lo.u32 %0, %0, %1, 0x1CE4E5B9;" : "+r"(a[k]) : "r"(b[k]));
+      }
+      if (KIND == 3) {
+        asm volatile("mad.hi.u32 %0, %0, %1, 0x7F4A7C15;" : "+r"(b[k]) : "r"(a[k]));
+        asm volatile("mad.hi.u32 %0, %0, %1, 0x1CE4E5B9;" : "+r"(a[k]) : "r"(b[k]));
+      }
+      if (KIND == 4) {
+        asm volatile("{\n\t.reg .u64 w;\n\tmad.wide.u32 w, %0, %1, %2;\n\tcvt.u32.u64 %0, w;\n\t}"
+                     : "+r"(b[k]) : "r"(a[k]), "l"((uint64_t)a[k]));
+        asm volatile("{\n\t.reg .u64 w;\n\tmad.wide.u32 w, %0, %1, %2;\n\tcvt.u32.u64 %0, w;\n\t}"
+                     : "+r"(a[k]) : "r"(b[k]), "l"((uint64_t)b[k]));
       }
     }
   }
@@ -66,18 +79,20 @@ __global__ void __launch_bounds__(kProbeThreads)
 
 }  // namespace
 
-// Launch one probe on `stream`: kind 0, 1 or 2 (see above), `iters` steps,
+// Launch one probe on `stream`: kind 0 .. 4 (see above), `iters` steps,
 // `grid` CTAs of 1024 threads.  sink: device, grid x 1024 uint32 (written);
 // clocks: device, 3 x grid uint64 (written: per CTA its SM id and the SM
 // clock counter at the start and the end of its loop).  Returns 0 or a
-// cudaError_t value.  Lane-ops per CTA: 1024 x iters x 8 x (2, 2 or 4).
+// cudaError_t value.  Lane-ops per CTA: 1024 x iters x 8 x (4 for kind 2, else 2).
 APC_PROBE_EXPORT int apc_probe_int_rate(int kind, uint32_t iters, uint32_t grid, uint32_t *sink,
                                         unsigned long long *clocks, void *stream) {
-  if (kind < 0 || kind > 2 || grid == 0 || !sink || !clocks) return (int)cudaErrorInvalidValue;
+  if (kind < 0 || kind > 4 || grid == 0 || !sink || !clocks) return (int)cudaErrorInvalidValue;
   cudaStream_t s = (cudaStream_t)stream;
   if (kind == 0) int_rate_kernel<0><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
   else if (kind == 1) int_rate_kernel<1><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
-  else int_rate_kernel<2><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
+  else if (kind == 2) int_rate_kernel<2><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
+  else if (kind == 3) int_rate_kernel<3><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
+  else int_rate_kernel<4><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, sink, clocks);
   return (int)cudaGetLastError();
 }
 

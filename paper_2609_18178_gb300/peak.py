@@ -15,8 +15,8 @@ import statistics
 
 from . import _build
 
-KINDS = {"alu": 0, "fma": 1, "both": 2}
-OPS_PER_STEP = {"alu": 2, "fma": 2, "both": 4}
+KINDS = {"alu": 0, "fma": 1, "both": 2, "mulhi": 3, "mulwide": 4}
+OPS_PER_STEP = {"alu": 2, "fma": 2, "both": 4, "mulhi": 2, "mulwide": 2}
 
 _lib = None
 
@@ -34,10 +34,11 @@ def library():
     return _lib
 
 
-def int_rates(iters: int = 8192, reps: int = 5) -> dict:
+def int_rates(iters: int = 8192, reps: int = 5, kinds=("alu", "fma", "both")) -> dict:
     """Lane-op rates of the ALU pipe ("alu": funnel shifts and xors), the
     multiply-add pipe ("fma": 32-bit multiply-adds) and both together
-    ("both": equal numbers, the issue-limited mix), on a grid of one
+    ("both": equal numbers, the issue-limited mix), and on request of the
+    high ("mulhi") and widening ("mulwide") multiply-adds, on a grid of one
     1024-thread CTA per SM; median of ``reps`` launches after one warm-up.
     Per clock: each SM's lane-ops over the span of its SM clock counter from
     its first CTA's start to its last CTA's end, median over the SMs."""
@@ -51,7 +52,8 @@ def int_rates(iters: int = 8192, reps: int = 5) -> dict:
     clocks = torch.empty(3 * grid, dtype=torch.int64, device="cuda")
     stream = torch.cuda.current_stream()
     out = {"sms": sms, "grid": grid, "threads": threads, "iters": iters}
-    for name, kind in KINDS.items():
+    for name in kinds:
+        kind = KINDS[name]
         per_cta = threads * iters * chains * OPS_PER_STEP[name]
         clk, sec = [], []
         for r in range(reps + 1):
