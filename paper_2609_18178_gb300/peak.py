@@ -25,7 +25,7 @@ def library():
     global _lib
     if _lib is None:
         lib = ctypes.CDLL(_build.build_probe())
-        lib.apc_probe_int_rate.argtypes = [ctypes.c_int, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_void_p,
+        lib.apc_probe_int_rate.argtypes = [ctypes.c_int, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32,
                                            ctypes.c_void_p, ctypes.c_void_p]
         lib.apc_probe_int_rate.restype = ctypes.c_int
         lib.apc_probe_threads.restype = ctypes.c_int
@@ -48,8 +48,7 @@ def int_rates(iters: int = 8192, reps: int = 5, kinds=("alu", "fma", "both")) ->
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     grid = sms
     threads, chains = lib.apc_probe_threads(), lib.apc_probe_chains()
-    sink = torch.empty(grid * threads, dtype=torch.int32, device="cuda")
-    clocks = torch.empty(3 * grid, dtype=torch.int64, device="cuda")
+    clocks = torch.empty(3 * grid + 1, dtype=torch.int64, device="cuda")
     stream = torch.cuda.current_stream()
     out = {"sms": sms, "grid": grid, "threads": threads, "iters": iters}
     for name in kinds:
@@ -59,8 +58,8 @@ def int_rates(iters: int = 8192, reps: int = 5, kinds=("alu", "fma", "both")) ->
         for r in range(reps + 1):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            rc = lib.apc_probe_int_rate(kind, iters, grid, ctypes.c_void_p(sink.data_ptr()),
-                                        ctypes.c_void_p(clocks.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
+            rc = lib.apc_probe_int_rate(kind, iters, grid, 0x5EED5EED, ctypes.c_void_p(clocks.data_ptr()),
+                                        ctypes.c_void_p(stream.cuda_stream))
             if rc:
                 raise RuntimeError("integer-rate probe launch failed (cudaError %d)" % rc)
             e1.record(stream)
