@@ -511,12 +511,17 @@ def run_gpu(args):
     # stream; later steps update the state in place.
     first_digests = apc.digests_to_host(apc.commit_step(tab, step_t, HP, stream=s, out=out_c))
 
+    user_limit = os.environ.get("APC_GRID_LIMIT")
+
     def grid_limit(n):
-        # APC_GRID_LIMIT is read by every library call (include/apc.h)
+        # APC_GRID_LIMIT is read by every library call (include/apc.h); 0
+        # restores whatever the caller of the bench had set
         if n:
             os.environ["APC_GRID_LIMIT"] = str(n)
-        else:
+        elif user_limit is None:
             os.environ.pop("APC_GRID_LIMIT", None)
+        else:
+            os.environ["APC_GRID_LIMIT"] = user_limit
 
     def one_step(ev=None):
         if ev is not None:
@@ -878,7 +883,7 @@ def run_gpu(args):
                              % (n_commit_launches, n_digest_launches, len(entries), len(vbufs)),
         "digests": ["%016x" % d for d in whole_d],
         "first_commit_digests": ["%016x" % d for d in first_whole],
-        "oracle_parity": (None if oracle_c5 is None or w.name != "c5" or world != 1 else
+        "oracle_parity": (None if oracle_c5 is None or whole.name != "c5" or world != 1 else
                           {"workload": "c5", "step": step_t,
                            "gpu_first_commit_digests": ["%016x" % d for d in first_digests],
                            "oracle_digests": ["%016x" % d for d in oracle_c5],
