@@ -46,6 +46,53 @@ __device__ __forceinline__ uint32_t adamw_element(float &p, float &m, float &v, 
   return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(pn));
 }
 
+// Two binary32 values in one 64-bit register pair, lane 0 in the low half,
+// for the packed two-lane multiply (mul.rn.f32x2): each lane is an IEEE
+// binary32 multiply rounded to nearest even, subnormals kept, so it gives
+// each lane the bits of the scalar multiply.
+__device__ __forceinline__ uint64_t pack2(float a, float b) {
+  return ((uint64_t)__float_as_uint(b) << 32) | __float_as_uint(a);
+}
+__device__ __forceinline__ float lane0(uint64_t x) { return __uint_as_float((uint32_t)x); }
+__device__ __forceinline__ float lane1(uint64_t x) { return __uint_as_float((uint32_t)(x >> 32)); }
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// adamw_element for two elements at once: the same binary32 operations in
+// the same order, each multiply issued as one packed two-lane instruction.
+// The adds and the subtract stay scalar __fadd_rn / __fsub_rn: a packed
+// product feeding a packed add was found contracted into a fused
+// multiply-add by the assembler (a 1-ulp change in a quarter of the
+// elements), while the scalar round-to-nearest adds are never fused.  The
+// square root and the divide run per lane.  w0, w1: the bf16 bits of p'.
+__device__ __forceinline__ void adamw_pair(float &p0, float &p1, float &m0, float &m1, float &v0, float &v1,
+                                           uint32_t g16a, uint32_t g16b, const Scalars &s, uint32_t &w0,
+                                           uint32_t &w1) {
+  const uint64_t g = pack2(__uint_as_float(g16a << 16), __uint_as_float(g16b << 16));
+  const uint64_t t1 = mul2(pack2(s.h[0], s.h[0]), pack2(m0, m1));
+  const uint64_t t2 = mul2(pack2(s.h[1], s.h[1]), g);
+  const uint64_t gg = mul2(g, g);
+  const uint64_t t3 = mul2(pack2(s.h[2], s.h[2]), pack2(v0, v1));
+  const uint64_t t4 = mul2(pack2(s.h[3], s.h[3]), gg);
+  const float mn0 = __fadd_rn(lane0(t1), lane0(t2)), mn1 = __fadd_rn(lane1(t1), lane1(t2));
+  const float vn0 = __fadd_rn(lane0(t3), lane0(t4)), vn1 = __fadd_rn(lane1(t3), lane1(t4));
+  const uint64_t t5 = mul2(pack2(__fsqrt_rn(vn0), __fsqrt_rn(vn1)), pack2(s.h[7], s.h[7]));
+  const float den0 = __fadd_rn(lane0(t5), s.h[4]), den1 = __fadd_rn(lane1(t5), s.h[4]);
+  const uint64_t t6 = mul2(pack2(p0, p1), pack2(s.h[5], s.h[5]));
+  const uint64_t t7 = mul2(pack2(s.h[6], s.h[6]), pack2(__fdiv_rn(mn0, den0), __fdiv_rn(mn1, den1)));
+  p0 = __fsub_rn(lane0(t6), lane0(t7));
+  p1 = __fsub_rn(lane1(t6), lane1(t7));
+  m0 = mn0;
+  m1 = mn1;
+  v0 = vn0;
+  v1 = vn1;
+  w0 = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(p0));
+  w1 = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(p1));
+}
+
 // The two 64-bit multiplies of the splitmix64 finaliser, z * C mod 2^64 for
 // a constant C = (chi : clo), in one of two instruction forms.  Which one is
 // faster depends on the kernel around it (both give the same bits):

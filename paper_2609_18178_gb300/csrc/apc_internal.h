@@ -70,6 +70,11 @@ constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
 #ifndef APC_SMEM_CARVEOUT
 #define APC_SMEM_CARVEOUT -1
 #endif
+// AdamW's multiplies as packed two-lane binary32 instructions over pairs of
+// elements (1), or one element at a time (0); the bits are the same.
+#ifndef APC_PAIRED_ADAMW
+#define APC_PAIRED_ADAMW 1
+#endif
 // A stage holds one tile of p, m, v and g: 14 bytes per element for fp32
 // state (133 KB per CTA at the defaults), 8 for bf16 state (162 KB).
 
