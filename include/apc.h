@@ -32,6 +32,10 @@
  *              den = sqrt(v') * rsb2 + eps          (IEEE sqrt)
  *              p' = p*(1-lr*wd) - step*(m'/den)     (IEEE divide)
  *              w  = bf16 round-to-nearest-even of p'
+ *            Infinities and NaNs in p, m, v or g follow IEEE 754 through
+ *            each operation.  A NaN result is written as a NaN whose payload
+ *            is left open (IEEE 754 does not fix it), and the bf16 copy of a
+ *            NaN is a bf16 NaN; every other result is the exact bits above.
  *   digest   D_B = sum over elements of
  *              splitmix64(((G mod 2^32) << 32) | bits_B)   (mod 2^64)
  *            G the element's index in the flat model (global_offset + i),

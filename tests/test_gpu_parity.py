@@ -545,6 +545,79 @@ def test_hyperparameters_and_edge_values(hp, step):
     assert_same(*run_small([adversarial(40000, step), adversarial(333, step + 1)], step, hp))
 
 
+F32_NAN = np.array([0x7FC00000, 0xFFC00000, 0x7F800001, 0x7FFFFFFF], np.uint32).view(np.float32)
+BF16_NAN = np.array([0x7FC0, 0xFFC0, 0x7F81, 0xFFFF], np.uint16)
+
+
+def nonfinite(n, seed):
+    """Generated state with non-finite inputs: blocks of infinite and NaN
+    gradients, parameters and moments and of negative second moments (whose
+    square root is NaN), then single non-finite values scattered over the
+    rest, so that packed pairs and vectors mix NaN and finite lanes."""
+    rng = np.random.default_rng(seed)
+    t = gen(n, seed * n, seed + 1)
+    p, m, v, g = t["p"], t["m"], t["v"], t["g"]
+    k = n // 12
+    inf = np.array([np.inf, -np.inf], np.float32)
+    g[:k] = rng.choice(np.array([0x7F80, 0xFF80], np.uint16), k)
+    g[k:2 * k] = rng.choice(BF16_NAN, k)
+    p[2 * k:3 * k] = rng.choice(inf, k)
+    p[3 * k:4 * k] = rng.choice(F32_NAN, k)
+    m[4 * k:5 * k] = rng.choice(inf, k)
+    m[5 * k:6 * k] = rng.choice(F32_NAN, k)
+    v[6 * k:7 * k] = np.inf
+    v[7 * k:8 * k] = rng.choice(F32_NAN, k)
+    v[8 * k:9 * k] = -np.abs(v[8 * k:9 * k]) - np.float32(1e-3)
+    rest = np.arange(9 * k, n)
+    for a, pool in ((p, np.concatenate([inf, F32_NAN])), (m, np.concatenate([inf, F32_NAN])),
+                    (v, np.concatenate([inf[:1], F32_NAN])), (g, np.concatenate([np.array([0x7F80, 0xFF80],
+                                                                                     np.uint16), BF16_NAN]))):
+        at = rest[rng.random(rest.size) < 0.03]
+        a[at] = rng.choice(pool, at.size)
+    return t
+
+
+def assert_same_up_to_nan_payload(devs, ref):
+    """Every result that is not NaN bit-identical to the oracle's; NaN exactly
+    where the oracle's is NaN (IEEE 754 leaves a NaN result's payload open,
+    and the GPU and the host CPUs pick different ones); the bf16 copy of a
+    NaN parameter is a bf16 NaN.  Returns the number of NaN parameters."""
+    nan_p = 0
+    for d, r in zip(devs, ref):
+        for k in "pmv":
+            a, b = host(d[k], np.uint32), r[k].view(np.uint32)
+            bn = np.isnan(r[k])
+            assert np.array_equal(np.isnan(a.view(np.float32)), bn), "%s: NaN positions differ" % k
+            bad = np.nonzero((a != b) & ~bn)[0]
+            assert bad.size == 0, "%s differs at %s: %s vs %s" % (k, bad[:5], a[bad[:5]], b[bad[:5]])
+        w, pn = host(d["w"], np.uint16), np.isnan(r["p"])
+        assert np.array_equal(w[~pn], r["w"][~pn]), "w differs"
+        assert np.all((w[pn] & 0x7FFF) > 0x7F80), "w of a NaN parameter is not a bf16 NaN"
+        nan_p += int(pn.sum())
+    return nan_p
+
+
+@pytest.mark.parametrize("step", [1, 18])
+def test_non_finite_inputs(step):
+    """Infinite and NaN inputs through the fp32 commit: results equal the
+    oracle's up to NaN payloads, infinities included.  The digests cannot be
+    the oracle's where a NaN was written, so they are checked against the
+    verification pass over the written buffers and against a second run."""
+    tensors = [nonfinite(40000, step), nonfinite(333, step + 7)]
+    runs = []
+    for _ in range(2):
+        devs, dgot, ref, _ = run_small([dict(t, p=t["p"].copy(), m=t["m"].copy(), v=t["v"].copy())
+                                        for t in tensors], step)
+        nan_p = assert_same_up_to_nan_payload(devs, ref)
+        assert 1000 < nan_p < 40333 - 10000          # both kinds of result are well represented
+        assert any(np.isinf(r["p"]).any() for r in ref) and any(np.isinf(r["v"]).any() for r in ref)
+        bufs = [b for d, t in zip(devs, tensors) for b in apc.state_buffers(d["p"], d["m"], d["v"], d["w"], t["goff"])]
+        assert apc.digests_to_host(apc.digest(bufs, 4)) == dgot
+        runs.append((dgot, [host(d[k], np.uint32).copy() for d in devs for k in "pmv"]))
+    assert runs[0][0] == runs[1][0]
+    assert all(np.array_equal(a, b) for a, b in zip(runs[0][1], runs[1][1]))
+
+
 def test_commit_zero_grad_reaches_committed_boundary():
     """With APC_COMMIT_ZERO_GRAD the same pass zeroes every gradient: outputs
     and digests equal the oracle's, the guard counts the oracle's nonzero
@@ -629,6 +702,36 @@ def run_bf16(tensors, step, hp=HP, zero_grad=False, shift=0):
         g_after = host(d["g"], np.uint16)[sl]
         assert (not g_after.any()) if zero_grad else np.array_equal(g_after, t["g"])
     assert apc.digests_to_host(out) == want
+
+
+def test_bf16_state_non_finite_inputs():
+    """Infinite and NaN bf16 words through the bf16-state commit.  Each result
+    is the binary32 step rounded once to bf16: where the fp32 oracle's result
+    on the widened inputs is NaN the word is a bf16 NaN, elsewhere it equals
+    the bf16 oracle's word; the digests equal the verification pass's."""
+    rng = np.random.default_rng(52)
+    n, step = 30011, 9
+    t = gen16(n, 5000, step)
+    specials = np.concatenate([np.array([0x7F80, 0xFF80], np.uint16), BF16_NAN])
+    for k in "pmvg":
+        at = rng.random(n) < 0.04
+        t[k][at] = rng.choice(specials, int(at.sum()))
+    t["v"][rng.random(n) < 0.02] |= 0x8000                         # negative second moments
+    d = {k: dev(t[k]) for k in "pmvg"}
+    out = apc.commit_step_bf16([apc.TensorEntryBF16(d["p"], d["m"], d["v"], d["g"], t["goff"])], step, HP)
+    got = apc.digests_to_host(out)
+    h8 = oracle.resolve_hparams(HP, step)
+    p, m, v = t["p"].copy(), t["m"].copy(), t["v"].copy()
+    oracle.commit_bf16(p, m, v, t["g"], t["goff"], h8)
+    p32, m32, v32 = gf32(t["p"]), gf32(t["m"]), gf32(t["v"])
+    oracle.adamw(p32, m32, v32, t["g"], h8)
+    for k, ref16, ref32 in (("p", p, p32), ("m", m, m32), ("v", v, v32)):
+        a, nan = host(d[k], np.uint16), np.isnan(ref32)
+        assert np.array_equal(a[~nan], ref16[~nan]), k
+        assert np.all((a[nan] & 0x7FFF) > 0x7F80), k
+        assert 0 < nan.sum() < n // 2, k
+    assert np.isinf(gf32(p)).any()
+    assert apc.digests_to_host(apc.digest(apc.state_buffers_bf16(d["p"], d["m"], d["v"], t["goff"]), 3)) == got
 
 
 # Elements per tile of the commit kernel's bf16-state layout (27 x 32 threads x 3 groups of 4).

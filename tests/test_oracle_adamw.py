@@ -8,7 +8,7 @@ against things other than itself:
 * the scalars against exact rational arithmetic on the decimal
   hyper-parameters (within one binary32 ulp),
 * the step-1 closed form (m = v = 0),
-* special cases (lr = 0, g = 0, beta1 = 0, wd = 0),
+* special cases (lr = 0, g = 0, beta1 = 0, wd = 0) and non-finite inputs,
 * the textbook form of AdamW evaluated in double, within a forward error
   bound derived from the number of binary32 roundings,
 * the bf16 copy against torch's float -> bfloat16 conversion,
@@ -224,6 +224,54 @@ def test_gradients_whose_square_overflows():
     assert np.all(np.isposinf(v))
     assert np.array_equal(p.view(np.uint32), p_dec.view(np.uint32))
     assert np.all(np.abs(m - m1) <= bm + 2.0 ** -149)
+
+
+INF, NAN = np.float32(np.inf), np.float32(np.nan)
+
+
+def test_non_finite_values_propagate_as_ieee_says():
+    """One non-finite input per element, the other three finite, against what
+    IEEE 754 fixes for each operation of the step (inf - inf, inf / inf and
+    the square root of a negative are NaN; a finite value times a positive
+    scalar keeps an infinity's sign).  The unaffected moments equal those of
+    the same element with every input finite."""
+    p0, m0, v0, g0 = 0.5, 0.01, 1e-4, 0x3E80          # g0 = bf16 0.25
+    cases = [  # (p, m, v, g bits) -> (p', m', v') with None for "as the finite element"
+        ((p0, m0, v0, 0x7F80), ("nan", INF, INF)),
+        ((p0, m0, v0, 0xFF80), ("nan", -INF, INF)),
+        ((p0, m0, v0, 0x7FC1), ("nan", "nan", "nan")),
+        ((INF, m0, v0, g0), (INF, None, None)),
+        ((-INF, m0, v0, g0), (-INF, None, None)),
+        ((NAN, m0, v0, g0), ("nan", None, None)),
+        ((p0, INF, v0, g0), (-INF, INF, None)),
+        ((p0, -INF, v0, g0), (INF, -INF, None)),
+        ((p0, NAN, v0, g0), ("nan", "nan", None)),
+        ((p0, m0, INF, g0), ("decay", None, INF)),
+        ((p0, m0, NAN, g0), ("nan", None, "nan")),
+        ((p0, m0, -1.0, g0), ("nan", None, "negative")),
+    ]
+    n = len(cases) + 1
+    p = np.array([c[0][0] for c in cases] + [p0], np.float32)
+    m = np.array([c[0][1] for c in cases] + [m0], np.float32)
+    v = np.array([c[0][2] for c in cases] + [v0], np.float32)
+    g = np.array([c[0][3] for c in cases] + [g0], np.uint16)
+    h = oracle.resolve_hparams(HP, 5)
+    w = oracle.adamw(p, m, v, g, h)
+    fin = dict(m=m[n - 1], v=v[n - 1])
+    for i, (_, want) in enumerate(cases):
+        for k, got, wv in (("p", p[i], want[0]), ("m", m[i], want[1]), ("v", v[i], want[2])):
+            if wv is None:
+                assert got.view(np.uint32) == fin[k].view(np.uint32), (i, k)
+            elif wv == "nan":
+                assert np.isnan(got), (i, k)
+            elif wv == "decay":      # u = m' / inf = 0, so p' = p (1 - lr wd), one product
+                assert got == np.float32(p0) * h[5], (i, k)
+            elif wv == "negative":   # b2 v + (1 - b2) g^2 < 0: finite, and its square root is NaN
+                assert np.isfinite(got) and got < 0, (i, k)
+            else:
+                assert got == wv, (i, k, got)
+        if np.isinf(p[i]):           # the bf16 copy of an infinity is the same infinity
+            assert w[i] == (0x7F80 if p[i] > 0 else 0xFF80), i
 
 
 def test_bounds_would_catch_plausible_mistakes():
