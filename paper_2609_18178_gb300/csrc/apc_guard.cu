@@ -6,9 +6,9 @@
 //
 // A word counts when its bit pattern is nonzero (so a -0.0 gradient counts).
 // The pass reads 4 (fp32) or 2 (bf16) bytes per element and does one compare
-// per element, so it is bound by HBM.  Same buffer plans and tiling as the
-// digest kernel (apc_digest.cu): 16-byte aligned bodies in tiles of
-// kDigestTile elements over a persistent grid, loads issued for the whole
+// per element, so it is bound by HBM.  Same buffer plans and tiling scheme as
+// the digest kernel (apc_digest.cu), with its own shape: 16-byte aligned
+// bodies in tiles of kCountTile elements over a persistent grid, loads issued for the whole
 // tile before counting, scalar head and tail by the CTA that owns the first
 // tile, per-slot running counts flushed on CTA-uniform slot changes.
 #include <cuda_runtime.h>
@@ -36,7 +36,7 @@ __device__ __forceinline__ uint32_t nz16(uint32_t w) {
 }
 
 template <int MAXE>
-__global__ void __launch_bounds__(kThreads) count_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
+__global__ void __launch_bounds__(kCountThreads) count_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
                                                          unsigned long long *out) {
   __shared__ unsigned long long s_acc[APC_MAX_SLOTS];
   if (threadIdx.x < APC_MAX_SLOTS) s_acc[threadIdx.x] = 0;
@@ -54,15 +54,15 @@ __global__ void __launch_bounds__(kThreads) count_kernel(const __grid_constant__
     const uint64_t local = tile - E.tile_begin;
     const uint64_t head = E.head;
     const uint64_t vec_end = head + ((E.n - head) & ~(uint64_t)(kVec - 1));
-    const uint64_t base = head + local * kDigestTile;
+    const uint64_t base = head + local * kCountTile;
     uint32_t c = 0;
     if (E.dtype == 0) {
       const uint32_t *d = reinterpret_cast<const uint32_t *>(E.data);
-      uint4 x[kDigestUnroll][2];
-      bool ok[kDigestUnroll];
+      uint4 x[kCountUnroll][2];
+      bool ok[kCountUnroll];
 #pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u) {
-        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
+      for (int u = 0; u < kCountUnroll; ++u) {
+        const uint64_t i = base + (uint64_t)(u * kCountThreads + threadIdx.x) * kVec;
         ok[u] = i < vec_end;
         if (ok[u]) {
           x[u][0] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
@@ -70,20 +70,20 @@ __global__ void __launch_bounds__(kThreads) count_kernel(const __grid_constant__
         }
       }
 #pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u)
+      for (int u = 0; u < kCountUnroll; ++u)
         if (ok[u]) c += nz32(x[u][0]) + nz32(x[u][1]);
     } else {
       const uint16_t *d = reinterpret_cast<const uint16_t *>(E.data);
-      uint4 x[kDigestUnroll];
-      bool ok[kDigestUnroll];
+      uint4 x[kCountUnroll];
+      bool ok[kCountUnroll];
 #pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u) {
-        const uint64_t i = base + (uint64_t)(u * kThreads + threadIdx.x) * kVec;
+      for (int u = 0; u < kCountUnroll; ++u) {
+        const uint64_t i = base + (uint64_t)(u * kCountThreads + threadIdx.x) * kVec;
         ok[u] = i < vec_end;
         if (ok[u]) x[u] = __ldcs(reinterpret_cast<const uint4 *>(d + i));
       }
 #pragma unroll
-      for (int u = 0; u < kDigestUnroll; ++u)
+      for (int u = 0; u < kCountUnroll; ++u)
         if (ok[u]) c += nz16(x[u].x) + nz16(x[u].y) + nz16(x[u].z) + nz16(x[u].w);
     }
     if (local == 0) {
@@ -108,18 +108,18 @@ __global__ void __launch_bounds__(kThreads) count_kernel(const __grid_constant__
 }  // namespace
 
 int launch_count_small(const DigestPlan<kDigestSmall> &plan, unsigned grid, void *stream, unsigned long long *out) {
-  count_kernel<kDigestSmall><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
+  count_kernel<kDigestSmall><<<grid, kCountThreads, 0, (cudaStream_t)stream>>>(plan, out);
   return (int)cudaGetLastError();
 }
 
 int launch_count_large(const DigestPlan<kDigestLarge> &plan, unsigned grid, void *stream, unsigned long long *out) {
-  count_kernel<kDigestLarge><<<grid, kThreads, 0, (cudaStream_t)stream>>>(plan, out);
+  count_kernel<kDigestLarge><<<grid, kCountThreads, 0, (cudaStream_t)stream>>>(plan, out);
   return (int)cudaGetLastError();
 }
 
 int count_blocks_per_sm(bool large, int *out) {
-  cudaError_t e = large ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, count_kernel<kDigestLarge>, kThreads, 0)
-                        : cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, count_kernel<kDigestSmall>, kThreads, 0);
+  cudaError_t e = large ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, count_kernel<kDigestLarge>, kCountThreads, 0)
+                        : cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, count_kernel<kDigestSmall>, kCountThreads, 0);
   return (int)e;
 }
 

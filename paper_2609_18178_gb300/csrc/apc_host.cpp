@@ -392,9 +392,10 @@ APC_EXPORT apc_status apc_commit_step_bf16(const apc_tensor_bf16 *table, int32_t
 
 namespace {
 
-// Validate a buffer list and turn it into digest/count plan entries.
+// Validate a buffer list and turn it into digest/count plan entries for a
+// kernel whose tiles hold `tile` elements.
 apc_status buffer_entries(const apc_buffer *bufs, int32_t num_bufs, int32_t num_slots, uint64_t *out,
-                          std::vector<apc::DigestEntry> *entries) {
+                          uint64_t tile, std::vector<apc::DigestEntry> *entries) {
   if (num_bufs < 0) return fail(APC_EINVAL, "num_bufs %d < 0", num_bufs);
   if (num_bufs > 0 && !bufs) return fail(APC_EINVAL, "bufs pointer is null");
   if (num_slots < 1 || num_slots > APC_MAX_SLOTS)
@@ -428,7 +429,7 @@ apc_status buffer_entries(const apc_buffer *bufs, int32_t num_bufs, int32_t num_
     e.slot = (uint8_t)b.slot;
     e.pad_ = 0;
     const uint64_t body = (b.n - e.head) / apc::kVec * apc::kVec;
-    e.tile_begin = std::max<uint64_t>(1, ceil_div(body, apc::kDigestTile));  // tile count until placed
+    e.tile_begin = std::max<uint64_t>(1, ceil_div(body, tile));  // tile count until placed
     entries->push_back(e);
   }
   const uintptr_t o = (uintptr_t)out;
@@ -444,7 +445,7 @@ APC_EXPORT apc_status apc_digest(const apc_buffer *bufs, int32_t num_bufs, int32
                                  uint64_t *out_digests) {
   g_last_error[0] = 0;
   std::vector<apc::DigestEntry> entries;
-  apc_status st = buffer_entries(bufs, num_bufs, num_slots, out_digests, &entries);
+  apc_status st = buffer_entries(bufs, num_bufs, num_slots, out_digests, apc::kDigestTile, &entries);
   if (st != APC_OK) return st;
   int e = (int)cudaMemsetAsync(out_digests, 0, (size_t)num_slots * sizeof(uint64_t), (cudaStream_t)stream);
   if (e) return cuda_fail(e, "cudaMemsetAsync(out_digests)");
@@ -463,7 +464,7 @@ APC_EXPORT apc_status apc_count_nonzero(const apc_buffer *bufs, int32_t num_bufs
                                         apc_stream_t stream, uint64_t *out_counts) {
   g_last_error[0] = 0;
   std::vector<apc::DigestEntry> entries;
-  apc_status st = buffer_entries(bufs, num_bufs, num_slots, out_counts, &entries);
+  apc_status st = buffer_entries(bufs, num_bufs, num_slots, out_counts, apc::kCountTile, &entries);
   if (st != APC_OK) return st;
   int e = (int)cudaMemsetAsync(out_counts, 0, (size_t)num_slots * sizeof(uint64_t), (cudaStream_t)stream);
   if (e) return cuda_fail(e, "cudaMemsetAsync(out_counts)");

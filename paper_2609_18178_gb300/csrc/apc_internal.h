@@ -123,18 +123,32 @@ constexpr int kCommitLarge = 440;
 static_assert(sizeof(CommitEntry) == 72, "entry layout");
 static_assert(sizeof(CommitPlan<kCommitLarge>) <= 32764, "kernel parameter limit");
 
-// Digest kernel: register-staged streaming (the pass is bound by integer
-// issue, so the loads are issued straight from the compute warps: a thread
-// handles kDigestUnroll 8-element vectors per tile).
+// Digest kernel: the loads are issued by the compute warps themselves (the
+// pass is bound by integer issue): a thread handles kDigestUnroll 8-element
+// vectors per tile.  512 threads put 8 warps on each of an SM's four
+// schedulers at two CTAs per SM; shapes that load the schedulers unevenly
+// (11 or 13 warps per CTA) run about 8% slower.
 #ifndef APC_DIGEST_THREADS
-#define APC_DIGEST_THREADS 384
+#define APC_DIGEST_THREADS 512
 #endif
 #ifndef APC_DIGEST_UNROLL
-#define APC_DIGEST_UNROLL 3
+#define APC_DIGEST_UNROLL 2
 #endif
 constexpr int kThreads = APC_DIGEST_THREADS;     // threads per CTA of the digest kernel
 constexpr int kDigestUnroll = APC_DIGEST_UNROLL; // thread-vectors per thread per tile
-constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 9,216 elements
+constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 8,192 elements
+
+// Guard (count) kernel: the same plans and tiling scheme with its own shape;
+// one compare per word leaves it bound by HBM.
+#ifndef APC_COUNT_THREADS
+#define APC_COUNT_THREADS 384
+#endif
+#ifndef APC_COUNT_UNROLL
+#define APC_COUNT_UNROLL 3
+#endif
+constexpr int kCountThreads = APC_COUNT_THREADS;
+constexpr int kCountUnroll = APC_COUNT_UNROLL;
+constexpr uint64_t kCountTile = (uint64_t)kCountThreads * kVec * kCountUnroll;  // 9,216 elements
 // Minimum resident CTAs per SM the digest kernel is compiled for (its
 // register cap: 65,536 / (threads x this)), and extra dynamic shared memory
 // per CTA beyond its stages (0 by default; a larger CTA footprint keeps two
@@ -148,7 +162,8 @@ constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 
 
 // One buffer of the digest kernel (32 bytes).
 //   head: scalar elements before the first 16-byte boundary (<= 7); then
-//         8-element vectors in tiles of kDigestTile; then a scalar tail, done
+//         8-element vectors in tiles of kDigestTile (kCountTile for the
+//         count kernel); then a scalar tail, done
 //         by the CTA that owns the buffer's first tile.
 struct DigestEntry {
   const void *data;

@@ -254,9 +254,11 @@ def test_digest_of_arbitrary_buffers():
     assert apc.digests_to_host(out) == want
 
 
-# Elements per tile of the verification kernel (384 threads x 3 vectors of 8):
-# every tile of a buffer but its last runs without bounds checks.
-DIGEST_TILE = 9216
+# Elements per tile of the verification kernel (512 threads x 2 vectors of 8)
+# and of the guard kernel (384 x 3): every tile of a buffer but its last runs
+# without bounds checks.
+DIGEST_TILE = 8192
+COUNT_TILE = 9216
 
 
 @pytest.mark.parametrize("limit", [None, 1, 5])
@@ -271,7 +273,7 @@ def test_digest_buffers_at_tile_boundaries(monkeypatch, limit):
         monkeypatch.setenv("APC_GRID_LIMIT", str(limit))
     rng = np.random.default_rng(33)
     bufs, each, keep = [], [], []
-    sizes = [k * DIGEST_TILE + d for k in (1, 2, 3) for d in (-8, -1, 0, 1, 7, 8, 9)] + [5 * DIGEST_TILE + 8 * 384]
+    sizes = [k * DIGEST_TILE + d for k in (1, 2, 3) for d in (-8, -1, 0, 1, 7, 8, 9)] + [5 * DIGEST_TILE + 8 * 512]
     for i, n in enumerate(sizes):
         for f32 in (True, False):
             shift = int(rng.integers(1, 8)) if i % 2 else 0   # a nonzero shift gives a scalar head
@@ -666,6 +668,27 @@ def test_count_nonzero_of_arbitrary_buffers():
         keep.append(t)
         bufs.append(apc.BufferEntry(t[shift:], slot, 0, apc.F32 if f32 else apc.BF16))
     assert apc.digests_to_host(apc.count_nonzero(bufs, 8)) == want
+
+
+def test_count_buffers_at_tile_boundaries():
+    """The guard kernel's own tiles: buffers whose bodies end on, just before
+    and just after its tile boundaries (and the verification kernel's), with
+    and without a scalar head, counted into four slots as numpy counts."""
+    rng = np.random.default_rng(34)
+    bufs, want, keep = [], [0] * 4, []
+    sizes = [k * t + d for t in (COUNT_TILE, DIGEST_TILE) for k in (1, 2) for d in (-8, -1, 0, 1, 9)]
+    for i, n in enumerate(sizes):
+        for f32 in (True, False):
+            shift = int(rng.integers(1, 8)) if i % 2 else 0
+            slot = (2 * i + f32) % 4
+            dt = np.uint32 if f32 else np.uint16
+            a = rng.integers(0, 2 ** (32 if f32 else 16), size=n + shift, dtype=np.uint64).astype(dt)
+            a[rng.random(n + shift) < 0.5] = 0
+            t = torch.from_numpy(a.view(np.int32 if f32 else np.int16)).cuda()
+            want[slot] += oracle.count_nonzero(a[shift:])
+            keep.append(t)
+            bufs.append(apc.BufferEntry(t[shift:], slot, 0, apc.F32 if f32 else apc.BF16))
+    assert apc.digests_to_host(apc.count_nonzero(bufs, 4)) == want
 
 
 # --------------------------------------------------------- bf16 state (f3)
