@@ -141,7 +141,7 @@ __device__ __forceinline__ void last_tile_ok(uint64_t base, uint64_t vec_end, bo
 // stg[(b * kStageSlots + k) * kThreads + t]: a warp's 16-byte reads of one
 // slot are contiguous.
 constexpr int kStageSlots = 2 * kDigestUnroll;                       // 16-byte words per thread per stage
-constexpr uint32_t kStageBytes = 2u * kStageSlots * kThreads * 16u;  // two stages: 65,536 bytes
+constexpr uint32_t kStageBytes = 2u * kStageSlots * kThreads * 16u;  // two stages: 131,072 bytes
 constexpr uint32_t kLaunchSmem = kStageBytes + APC_DIGEST_EXTRA_SMEM;
 
 __device__ __forceinline__ void cp16(uint32_t dst, const void *src) {
@@ -163,9 +163,9 @@ __device__ __forceinline__ uint32_t word_at(const DigestEntry &E, uint64_t i) {
                       : (uint32_t) reinterpret_cast<const uint16_t *>(E.data)[i];
 }
 
-// Two CTAs per SM (32 warps, 2 x 64 KB of stages), which caps the kernel at
-// 64 registers: a full tile's 16 terms per thread, without per-vector
-// checks, form one block that the compiler schedules within them.
+// One CTA per SM (32 warps, 128 KB of stages), which caps the kernel at 64
+// registers: a full tile's 16 terms per thread, without per-vector checks,
+// form one block that the compiler schedules within them.
 template <int MAXE>
 __global__ void __launch_bounds__(kThreads, APC_DIGEST_MIN_BLOCKS) digest_kernel(const __grid_constant__ DigestPlan<MAXE> plan,
                                                           unsigned long long *out) {

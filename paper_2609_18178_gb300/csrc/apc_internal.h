@@ -125,18 +125,19 @@ static_assert(sizeof(CommitPlan<kCommitLarge>) <= 32764, "kernel parameter limit
 
 // Digest kernel: the loads are issued by the compute warps themselves (the
 // pass is bound by integer issue): a thread handles kDigestUnroll 8-element
-// vectors per tile.  512 threads put 8 warps on each of an SM's four
-// schedulers at two CTAs per SM; shapes that load the schedulers unevenly
-// (11 or 13 warps per CTA) run about 8% slower.
+// vectors per tile.  One CTA of 1024 threads per SM puts 8 warps on each of
+// its four schedulers and gives each SM one contiguous run of tiles; two
+// CTAs of the same warps per SM run 2-3% slower, and shapes that load the
+// schedulers unevenly (11 or 13 warps per CTA) about 8% slower.
 #ifndef APC_DIGEST_THREADS
-#define APC_DIGEST_THREADS 512
+#define APC_DIGEST_THREADS 1024
 #endif
 #ifndef APC_DIGEST_UNROLL
 #define APC_DIGEST_UNROLL 2
 #endif
 constexpr int kThreads = APC_DIGEST_THREADS;     // threads per CTA of the digest kernel
 constexpr int kDigestUnroll = APC_DIGEST_UNROLL; // thread-vectors per thread per tile
-constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 8,192 elements
+constexpr uint64_t kDigestTile = (uint64_t)kThreads * kVec * kDigestUnroll;  // 16,384 elements
 
 // Guard (count) kernel: the same plans and tiling scheme with its own shape;
 // one compare per word leaves it bound by HBM.
@@ -154,7 +155,7 @@ constexpr uint64_t kCountTile = (uint64_t)kCountThreads * kVec * kCountUnroll;  
 // per CTA beyond its stages (0 by default; a larger CTA footprint keeps two
 // digest CTAs off one SM when another kernel is to share it).
 #ifndef APC_DIGEST_MIN_BLOCKS
-#define APC_DIGEST_MIN_BLOCKS 2
+#define APC_DIGEST_MIN_BLOCKS 1
 #endif
 #ifndef APC_DIGEST_EXTRA_SMEM
 #define APC_DIGEST_EXTRA_SMEM 0

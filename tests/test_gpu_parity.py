@@ -254,10 +254,10 @@ def test_digest_of_arbitrary_buffers():
     assert apc.digests_to_host(out) == want
 
 
-# Elements per tile of the verification kernel (512 threads x 2 vectors of 8)
+# Elements per tile of the verification kernel (1024 threads x 2 vectors of 8)
 # and of the guard kernel (384 x 3): every tile of a buffer but its last runs
 # without bounds checks.
-DIGEST_TILE = 8192
+DIGEST_TILE = 16384
 COUNT_TILE = 9216
 
 
@@ -273,7 +273,7 @@ def test_digest_buffers_at_tile_boundaries(monkeypatch, limit):
         monkeypatch.setenv("APC_GRID_LIMIT", str(limit))
     rng = np.random.default_rng(33)
     bufs, each, keep = [], [], []
-    sizes = [k * DIGEST_TILE + d for k in (1, 2, 3) for d in (-8, -1, 0, 1, 7, 8, 9)] + [5 * DIGEST_TILE + 8 * 512]
+    sizes = [k * DIGEST_TILE + d for k in (1, 2, 3) for d in (-8, -1, 0, 1, 7, 8, 9)] + [5 * DIGEST_TILE + 8 * 1024]
     for i, n in enumerate(sizes):
         for f32 in (True, False):
             shift = int(rng.integers(1, 8)) if i % 2 else 0   # a nonzero shift gives a scalar head
