@@ -255,10 +255,10 @@ def test_digest_of_arbitrary_buffers():
 
 
 # Elements per tile of the verification kernel (1024 threads x 2 vectors of 8)
-# and of the guard kernel (384 x 3): every tile of a buffer but its last runs
+# and of the guard kernel (1024 x 4): every tile of a buffer but its last runs
 # without bounds checks.
 DIGEST_TILE = 16384
-COUNT_TILE = 9216
+COUNT_TILE = 32768
 
 
 @pytest.mark.parametrize("limit", [None, 1, 5])
