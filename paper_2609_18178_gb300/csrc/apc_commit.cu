@@ -12,9 +12,10 @@
 // with +0 once its copy has landed: 2 more bytes per element.
 //
 // Warp-specialized pipeline (one persistent CTA per SM by default):
-//  * The producer warp walks the launch's tiles (L::kTile elements of one
-//    entry's 16-byte aligned body: 4,864 for fp32 state, 10,368 for bf16
-//    state) and, for each, waits until a ring stage is free and issues four
+//  * The producer warp walks the CTA's run of the launch's tiles (one
+//    contiguous run per CTA; a tile is L::kTile elements of one entry's
+//    16-byte aligned body: 4,864 for fp32 state, 10,368 for bf16 state)
+//    and, for each, waits until a ring stage is free and issues four
 //    bulk asynchronous copies -- p, m, v and g -- that complete on the
 //    stage's "full" mbarrier.  Loads never occupy consumer registers, and up
 //    to kCommitStages tiles per CTA are in flight.
@@ -333,6 +334,21 @@ __device__ __forceinline__ uint32_t find_tile(const CommitPlan<MAXE> &plan, uint
   return cur;
 }
 
+// This CTA's tiles: tile = t0, t0 + ts, ... while tile < t1 (the same walk
+// for the producer and the consumers).
+struct TileWalk {
+  uint64_t t0, t1, ts;
+};
+__device__ __forceinline__ TileWalk tile_walk(uint64_t total) {
+  const uint64_t b = blockIdx.x;
+  if (APC_COMMIT_CONTIGUOUS) {
+    const uint64_t per = total / gridDim.x, rem = total % gridDim.x;
+    const uint64_t t0 = b * per + (b < rem ? b : rem);
+    return {t0, t0 + per + (b < rem ? 1 : 0), 1};
+  }
+  return {b, total, gridDim.x};
+}
+
 template <class L, int MAXE, bool ZERO>
 __global__ void __launch_bounds__(L::kBoundThreads, kCommitBlocksPerSm)
     commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan, unsigned long long *out) {
@@ -362,7 +378,8 @@ __global__ void __launch_bounds__(L::kBoundThreads, kCommitBlocksPerSm)
       uint32_t cur = 0, phase = 0;
       int stage = 0;
       uint64_t issued = 0;
-      for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
+      const TileWalk w = tile_walk(plan.total_tiles);
+      for (uint64_t tile = w.t0; tile < w.t1; tile += w.ts) {
         if (*(volatile int *)&abort_flag) break;
         cur = find_tile(plan, cur, tile);
         const CommitEntry &E = plan.e[cur];
@@ -412,7 +429,8 @@ __global__ void __launch_bounds__(L::kBoundThreads, kCommitBlocksPerSm)
     const int ct = threadIdx.x;  // 0 .. L::kConsumers-1
     uint32_t phase = 0;
     int stage = 0;
-    for (uint64_t tile = blockIdx.x; tile < plan.total_tiles; tile += gridDim.x) {
+    const TileWalk w = tile_walk(plan.total_tiles);
+    for (uint64_t tile = w.t0; tile < w.t1; tile += w.ts) {
       if (!mbar_wait(&full[stage], phase)) {
         fail_wait(&abort_flag);
         break;

@@ -70,6 +70,12 @@ constexpr int kCommitBlocksPerSm = APC_COMMIT_BLOCKS_PER_SM;
 #ifndef APC_SMEM_CARVEOUT
 #define APC_SMEM_CARVEOUT -1
 #endif
+// Tile order of the commit kernel: 1 = CTA b takes one contiguous run of
+// tiles (the runs differ by at most one tile), 0.3-0.7% faster than 0 = CTA b
+// takes tiles b, b + grid, ... (the grid sweeping the table together).
+#ifndef APC_COMMIT_CONTIGUOUS
+#define APC_COMMIT_CONTIGUOUS 1
+#endif
 // AdamW's multiplies as packed two-lane binary32 instructions over pairs of
 // elements (1), or one element at a time (0); the bits are the same.
 #ifndef APC_PAIRED_ADAMW
