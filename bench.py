@@ -80,20 +80,24 @@ def integer_ceiling(words: dict, rates: dict) -> float:
     (``words``: count of fp32 and 16-bit words digested per element) fits
     the measured ALU and multiply-add lane rates and the issue width, with
     the flexible operations split between the two pipes as well as
-    possible (a convex piecewise-linear minimum, scanned finely)."""
+    possible (a convex piecewise-linear minimum, scanned finely).  The six
+    multiply-adds of a term's two 64-bit multiplies run at the measured rate
+    of whole 64-bit multiplies ("mul64", three multiply-adds each) when the
+    rates have it, else at the plain multiply-add rate."""
     A0 = sum(n * (t["alu_only"] + t["flex"] + t["funnel"]) for k, n in words.items() for t in [TERM_OPS[k]])
     F0 = sum(n * t["mul_only"] for k, n in words.items() for t in [TERM_OPS[k]])
     n1 = sum(n * TERM_OPS[k]["flex"] for k, n in words.items())
     nf = sum(n * TERM_OPS[k]["funnel"] for k, n in words.items())
     ra = rates["alu"]["lane_ops_per_clk_per_sm"]
     rf = rates["fma"]["lane_ops_per_clk_per_sm"]
+    rm = rates["mul64"]["lane_ops_per_clk_per_sm"] if "mul64" in rates else rf
     ri = ISSUE_LANES_PER_CLK_PER_SM
     best = None
     steps = 4000
     for i in range(steps + 1):
         x = (n1 + nf) * i / steps                    # operations moved to the multiply-add pipe
         extra = max(0.0, x - n1)                     # funnel shifts moved cost two multiply-adds each
-        t = max((A0 - x) / ra, (F0 + x + extra) / rf, (A0 + F0 + extra) / ri)
+        t = max((A0 - x) / ra, F0 / rm + (x + extra) / rf, (A0 + F0 + extra) / ri)
         best = t if best is None or t < best else best
     return 1.0 / best
 
@@ -128,9 +132,11 @@ def verify_roofline(rates, clk, n: int, v_ms: float, hbm_peak: float, launches: 
     bound, peak = ("alu", int_terms) if int_terms < hbm_terms else ("hbm", hbm_terms)
     rec.update(bound=bound, peak=peak / 1e12, frac=terms_per_s / peak, integer_peak=int_terms / 1e12,
                integer_frac=terms_per_s / int_terms, hbm_peak_terms=hbm_terms / 1e12,
-               measured_lane_ops_per_clk_per_sm={k: rates[k]["lane_ops_per_clk_per_sm"] for k in ("alu", "fma", "both")},
+               measured_lane_ops_per_clk_per_sm={k: rates[k]["lane_ops_per_clk_per_sm"]
+                                                 for k in ("alu", "fma", "both", "mul64") if k in rates},
                sm_mhz=sm_hz / 1e6,
-               peak_basis="splitmix64 as defined, 20 32-bit operations per term (6 xors on the ALU, 6 multiply-adds, "
+               peak_basis="splitmix64 as defined, 20 32-bit operations per term (6 xors on the ALU, the 6 "
+                          "multiply-adds of two 64-bit multiplies at the measured rate of whole 64-bit multiplies, "
                           "the adds and shifts on either pipe, a funnel shift costing two multiply-adds off the "
                           "ALU), split as well as possible over the ALU and multiply-add lane rates measured by "
                           "register-only probes (libapc_probe.so) and 128 issue lanes per clock per SM, at the "

@@ -9,8 +9,13 @@
 //   kind 2 (both): the two ALU operations and the two
 //          multiply-adds of kinds 0 and 1, interleaved          4 lane-ops
 //   kind 3 (high multiply): two 32-bit high multiply-adds     2 lane-ops
-//   kind 4 (wide multiply): two 32 x 32 -> 64-bit
-//          multiply-adds                                      2 lane-ops
+//   kind 4 (wide multiply, low half): two 32 x 32 -> 64-bit
+//          multiply-adds of which only the low half is used
+//          (so the assembler may issue a plain multiply-add)   2 lane-ops
+//   kind 5 (64-bit multiply): two 64 x 64 -> 64-bit multiplies,
+//          each counted as the three 32-bit multiply-adds that
+//          define it (the low halves' widening product, then the
+//          two cross products into the high word)             6 lane-ops
 // The operands of each operation come from the previous step, so the
 // compiler can neither fold nor hoist them.  Thread 0 of every CTA records
 // its SM's id and the SM clock counter when the CTA's loop starts and ends;
@@ -31,10 +36,13 @@ template <int KIND>
 __global__ void __launch_bounds__(kProbeThreads)
     int_rate_kernel(uint32_t iters, uint32_t seed, uint32_t marker, unsigned long long *clocks) {
   uint32_t a[kChains], b[kChains];
+  uint64_t w[kChains], v[kChains];
 #pragma unroll
   for (int k = 0; k < kChains; ++k) {
     a[k] = seed ^ (threadIdx.x * kChains + k);
     b[k] = a[k] * 0x9E3779B9u + 0x7F4A7C15u;
+    w[k] = ((uint64_t)b[k] << 32) | a[k] | 1u;
+    v[k] = ((uint64_t)a[k] << 32) | b[k] | 1u;
   }
   __syncthreads();
   const long long t0 = clock64();
@@ -54,6 +62,10 @@ __global__ void __launch_bounds__(kProbeThreads)
         asm volatile("mad.hi.u32 %0, %0, %1, 0x7F4A7C15;" : "+r"(b[k]) : "r"(a[k]));
         asm volatile("mad.hi.u32 %0, %0, %1, 0x1CE4E5B9;" : "+r"(a[k]) : "r"(b[k]));
       }
+      if (KIND == 5) {
+        asm volatile("mul.lo.u64 %0, %0, %1;" : "+l"(w[k]) : "l"(v[k]));
+        asm volatile("mul.lo.u64 %0, %0, %1;" : "+l"(v[k]) : "l"(w[k]));
+      }
       if (KIND == 4) {
         asm volatile("{\n\t.reg .u64 w;\n\tmad.wide.u32 w, %0, %1, %2;\n\tcvt.u32.u64 %0, w;\n\t}"
                      : "+r"(b[k]) : "r"(a[k]), "l"((uint64_t)a[k]));
@@ -68,7 +80,7 @@ __global__ void __launch_bounds__(kProbeThreads)
   // equal to the caller's marker makes (the compiler cannot rule it out).
   uint32_t x = 0;
 #pragma unroll
-  for (int k = 0; k < kChains; ++k) x ^= a[k] + b[k];
+  for (int k = 0; k < kChains; ++k) x ^= a[k] + b[k] + (uint32_t)(w[k] >> 32) + (uint32_t)(v[k] >> 32);
   if (x == marker) clocks[3 * gridDim.x] = x;
   if (threadIdx.x == 0) {
     uint32_t sm;
@@ -81,7 +93,7 @@ __global__ void __launch_bounds__(kProbeThreads)
 
 }  // namespace
 
-// Launch one probe on `stream`: kind 0 .. 4 (see above), `iters` steps,
+// Launch one probe on `stream`: kind 0 .. 5 (see above), `iters` steps,
 // `grid` CTAs of 1024 threads.  clocks: device, 3 x grid + 1 uint64 (written:
 // per CTA its SM id and the SM clock counter at the start and the end of its
 // loop; the last word only if some thread's result equals `marker`, which
@@ -89,13 +101,14 @@ __global__ void __launch_bounds__(kProbeThreads)
 // value.  Lane-ops per CTA: 1024 x iters x 8 x (4 for kind 2, else 2).
 APC_PROBE_EXPORT int apc_probe_int_rate(int kind, uint32_t iters, uint32_t grid, uint32_t marker,
                                         unsigned long long *clocks, void *stream) {
-  if (kind < 0 || kind > 4 || grid == 0 || !clocks) return (int)cudaErrorInvalidValue;
+  if (kind < 0 || kind > 5 || grid == 0 || !clocks) return (int)cudaErrorInvalidValue;
   cudaStream_t s = (cudaStream_t)stream;
   if (kind == 0) int_rate_kernel<0><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   else if (kind == 1) int_rate_kernel<1><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   else if (kind == 2) int_rate_kernel<2><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   else if (kind == 3) int_rate_kernel<3><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
-  else int_rate_kernel<4><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
+  else if (kind == 4) int_rate_kernel<4><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
+  else int_rate_kernel<5><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   return (int)cudaGetLastError();
 }
 

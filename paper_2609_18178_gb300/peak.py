@@ -15,8 +15,8 @@ import statistics
 
 from . import _build
 
-KINDS = {"alu": 0, "fma": 1, "both": 2, "mulhi": 3, "mulwide": 4}
-OPS_PER_STEP = {"alu": 2, "fma": 2, "both": 4, "mulhi": 2, "mulwide": 2}
+KINDS = {"alu": 0, "fma": 1, "both": 2, "mulhi": 3, "mulwide": 4, "mul64": 5}
+OPS_PER_STEP = {"alu": 2, "fma": 2, "both": 4, "mulhi": 2, "mulwide": 2, "mul64": 6}
 
 _lib = None
 
@@ -34,11 +34,13 @@ def library():
     return _lib
 
 
-def int_rates(iters: int = 8192, reps: int = 5, kinds=("alu", "fma", "both")) -> dict:
+def int_rates(iters: int = 8192, reps: int = 5, kinds=("alu", "fma", "both", "mul64")) -> dict:
     """Lane-op rates of the ALU pipe ("alu": funnel shifts and xors), the
-    multiply-add pipe ("fma": 32-bit multiply-adds) and both together
-    ("both": equal numbers, the issue-limited mix), and on request of the
-    high ("mulhi") and widening ("mulwide") multiply-adds, on a grid of one
+    multiply-add pipe ("fma": 32-bit multiply-adds), both together ("both":
+    equal numbers, the issue-limited mix) and whole 64-bit multiplies
+    ("mul64", three multiply-add lane-ops each), and on request of the
+    high ("mulhi") and widening ("mulwide", only the low half used)
+    multiply-adds, on a grid of one
     1024-thread CTA per SM; median of ``reps`` launches after one warm-up.
     Per clock: each SM's lane-ops over the span of its SM clock counter from
     its first CTA's start to its last CTA's end, median over the SMs."""

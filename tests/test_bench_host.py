@@ -42,6 +42,13 @@ def test_integer_ceiling_closed_forms():
     assert bench.integer_ceiling(words, rates(64, 1e-9 + 24 * 64 / 56)) == pytest.approx(64 / 56, rel=2e-2)
     # an ALU far faster than issue: issue binds at 80 operations
     assert bench.integer_ceiling(words, rates(1e6, 1e6)) == pytest.approx(128 / 80, rel=1e-6)
+    # 64-bit multiplies measured at full rate change nothing
+    full = dict(rates(64, 64), mul64={"lane_ops_per_clk_per_sm": 64})
+    assert bench.integer_ceiling(words, full) == pytest.approx(128 / 80, rel=1e-3)
+    # at half rate the 24 multiply-adds take 0.75 clocks; balance
+    # (56 - x) / 64 = 0.75 + x / 64 at x = 4 gives 52 / 64 clocks per element
+    half = dict(rates(64, 64), mul64={"lane_ops_per_clk_per_sm": 32})
+    assert bench.integer_ceiling(words, half) == pytest.approx(64 / 52, rel=1e-3)
 
 
 def test_reference_arm_reports_what_it_ran():
