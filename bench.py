@@ -82,15 +82,18 @@ def integer_ceiling(words: dict, rates: dict) -> float:
     the flexible operations split between the two pipes as well as
     possible (a convex piecewise-linear minimum, scanned finely).  The six
     multiply-adds of a term's two 64-bit multiplies run at the measured rate
-    of whole 64-bit multiplies ("mul64", three multiply-adds each) when the
-    rates have it, else at the plain multiply-add rate."""
+    of whole 64-bit multiplies, three multiply-adds each, in the faster of
+    the two forms probed ("mul64": the compiler's; "mul64x": one widening
+    and two plain multiply-adds) when the rates have them, else at the plain
+    multiply-add rate."""
     A0 = sum(n * (t["alu_only"] + t["flex"] + t["funnel"]) for k, n in words.items() for t in [TERM_OPS[k]])
     F0 = sum(n * t["mul_only"] for k, n in words.items() for t in [TERM_OPS[k]])
     n1 = sum(n * TERM_OPS[k]["flex"] for k, n in words.items())
     nf = sum(n * TERM_OPS[k]["funnel"] for k, n in words.items())
     ra = rates["alu"]["lane_ops_per_clk_per_sm"]
     rf = rates["fma"]["lane_ops_per_clk_per_sm"]
-    rm = rates["mul64"]["lane_ops_per_clk_per_sm"] if "mul64" in rates else rf
+    m64 = [rates[k]["lane_ops_per_clk_per_sm"] for k in ("mul64", "mul64x") if k in rates]
+    rm = max(m64) if m64 else rf
     ri = ISSUE_LANES_PER_CLK_PER_SM
     best = None
     steps = 4000
@@ -133,10 +136,10 @@ def verify_roofline(rates, clk, n: int, v_ms: float, hbm_peak: float, launches: 
     rec.update(bound=bound, peak=peak / 1e12, frac=terms_per_s / peak, integer_peak=int_terms / 1e12,
                integer_frac=terms_per_s / int_terms, hbm_peak_terms=hbm_terms / 1e12,
                measured_lane_ops_per_clk_per_sm={k: rates[k]["lane_ops_per_clk_per_sm"]
-                                                 for k in ("alu", "fma", "both", "mul64") if k in rates},
+                                                 for k in ("alu", "fma", "both", "mul64", "mul64x") if k in rates},
                sm_mhz=sm_hz / 1e6,
                peak_basis="splitmix64 as defined, 20 32-bit operations per term (6 xors on the ALU, the 6 "
-                          "multiply-adds of two 64-bit multiplies at the measured rate of whole 64-bit multiplies, "
+                          "multiply-adds of two 64-bit multiplies at the measured rate of whole 64-bit multiplies in their faster form, "
                           "the adds and shifts on either pipe, a funnel shift costing two multiply-adds off the "
                           "ALU), split as well as possible over the ALU and multiply-add lane rates measured by "
                           "register-only probes (libapc_probe.so) and 128 issue lanes per clock per SM, at the "

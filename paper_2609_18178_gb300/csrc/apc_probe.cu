@@ -16,6 +16,9 @@
 //          each counted as the three 32-bit multiply-adds that
 //          define it (the low halves' widening product, then the
 //          two cross products into the high word)             6 lane-ops
+//   kind 6 (64-bit multiply, explicit form): the same multiplies
+//          written as one widening and two 32-bit multiply-adds
+//          in the probe's own PTX                              6 lane-ops
 // The operands of each operation come from the previous step, so the
 // compiler can neither fold nor hoist them.  Thread 0 of every CTA records
 // its SM's id and the SM clock counter when the CTA's loop starts and ends;
@@ -66,6 +69,20 @@ __global__ void __launch_bounds__(kProbeThreads)
         asm volatile("mul.lo.u64 %0, %0, %1;" : "+l"(w[k]) : "l"(v[k]));
         asm volatile("mul.lo.u64 %0, %0, %1;" : "+l"(v[k]) : "l"(w[k]));
       }
+      if (KIND == 6) {
+        asm volatile("{\n\t.reg .u32 al, ah, bl, bh, rl, rh;\n\t"
+                     "mov.b64 {al, ah}, %0;\n\tmov.b64 {bl, bh}, %1;\n\t"
+                     "mul.wide.u32 %0, al, bl;\n\tmov.b64 {rl, rh}, %0;\n\t"
+                     "mad.lo.u32 rh, al, bh, rh;\n\tmad.lo.u32 rh, ah, bl, rh;\n\t"
+                     "mov.b64 %0, {rl, rh};\n\t}"
+                     : "+l"(w[k]) : "l"(v[k]));
+        asm volatile("{\n\t.reg .u32 al, ah, bl, bh, rl, rh;\n\t"
+                     "mov.b64 {al, ah}, %0;\n\tmov.b64 {bl, bh}, %1;\n\t"
+                     "mul.wide.u32 %0, al, bl;\n\tmov.b64 {rl, rh}, %0;\n\t"
+                     "mad.lo.u32 rh, al, bh, rh;\n\tmad.lo.u32 rh, ah, bl, rh;\n\t"
+                     "mov.b64 %0, {rl, rh};\n\t}"
+                     : "+l"(v[k]) : "l"(w[k]));
+      }
       if (KIND == 4) {
         asm volatile("{\n\t.reg .u64 w;\n\tmad.wide.u32 w, %0, %1, %2;\n\tcvt.u32.u64 %0, w;\n\t}"
                      : "+r"(b[k]) : "r"(a[k]), "l"((uint64_t)a[k]));
@@ -93,7 +110,7 @@ __global__ void __launch_bounds__(kProbeThreads)
 
 }  // namespace
 
-// Launch one probe on `stream`: kind 0 .. 5 (see above), `iters` steps,
+// Launch one probe on `stream`: kind 0 .. 6 (see above), `iters` steps,
 // `grid` CTAs of 1024 threads.  clocks: device, 3 x grid + 1 uint64 (written:
 // per CTA its SM id and the SM clock counter at the start and the end of its
 // loop; the last word only if some thread's result equals `marker`, which
@@ -101,14 +118,15 @@ __global__ void __launch_bounds__(kProbeThreads)
 // value.  Lane-ops per CTA: 1024 x iters x 8 x (4 for kind 2, else 2).
 APC_PROBE_EXPORT int apc_probe_int_rate(int kind, uint32_t iters, uint32_t grid, uint32_t marker,
                                         unsigned long long *clocks, void *stream) {
-  if (kind < 0 || kind > 5 || grid == 0 || !clocks) return (int)cudaErrorInvalidValue;
+  if (kind < 0 || kind > 6 || grid == 0 || !clocks) return (int)cudaErrorInvalidValue;
   cudaStream_t s = (cudaStream_t)stream;
   if (kind == 0) int_rate_kernel<0><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   else if (kind == 1) int_rate_kernel<1><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   else if (kind == 2) int_rate_kernel<2><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   else if (kind == 3) int_rate_kernel<3><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   else if (kind == 4) int_rate_kernel<4><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
-  else int_rate_kernel<5><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
+  else if (kind == 5) int_rate_kernel<5><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
+  else int_rate_kernel<6><<<grid, kProbeThreads, 0, s>>>(iters, 12345u, marker, clocks);
   return (int)cudaGetLastError();
 }
 

@@ -15,8 +15,8 @@ import statistics
 
 from . import _build
 
-KINDS = {"alu": 0, "fma": 1, "both": 2, "mulhi": 3, "mulwide": 4, "mul64": 5}
-OPS_PER_STEP = {"alu": 2, "fma": 2, "both": 4, "mulhi": 2, "mulwide": 2, "mul64": 6}
+KINDS = {"alu": 0, "fma": 1, "both": 2, "mulhi": 3, "mulwide": 4, "mul64": 5, "mul64x": 6}
+OPS_PER_STEP = {"alu": 2, "fma": 2, "both": 4, "mulhi": 2, "mulwide": 2, "mul64": 6, "mul64x": 6}
 
 _lib = None
 
@@ -34,11 +34,12 @@ def library():
     return _lib
 
 
-def int_rates(iters: int = 8192, reps: int = 5, kinds=("alu", "fma", "both", "mul64")) -> dict:
+def int_rates(iters: int = 8192, reps: int = 5, kinds=("alu", "fma", "both", "mul64", "mul64x")) -> dict:
     """Lane-op rates of the ALU pipe ("alu": funnel shifts and xors), the
     multiply-add pipe ("fma": 32-bit multiply-adds), both together ("both":
-    equal numbers, the issue-limited mix) and whole 64-bit multiplies
-    ("mul64", three multiply-add lane-ops each), and on request of the
+    equal numbers, the issue-limited mix) and whole 64-bit multiplies, three
+    multiply-add lane-ops each, in the compiler's form ("mul64") and as one
+    widening and two plain multiply-adds ("mul64x"), and on request of the
     high ("mulhi") and widening ("mulwide", only the low half used)
     multiply-adds, on a grid of one
     1024-thread CTA per SM; median of ``reps`` launches after one warm-up.

@@ -49,6 +49,9 @@ def test_integer_ceiling_closed_forms():
     # (56 - x) / 64 = 0.75 + x / 64 at x = 4 gives 52 / 64 clocks per element
     half = dict(rates(64, 64), mul64={"lane_ops_per_clk_per_sm": 32})
     assert bench.integer_ceiling(words, half) == pytest.approx(64 / 52, rel=1e-3)
+    # of two measured forms, the faster one counts
+    assert bench.integer_ceiling(words, dict(half, mul64x={"lane_ops_per_clk_per_sm": 64})) == \
+        pytest.approx(128 / 80, rel=1e-3)
 
 
 def test_reference_arm_reports_what_it_ran():
