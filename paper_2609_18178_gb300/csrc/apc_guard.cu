@@ -8,9 +8,10 @@
 // The pass reads 4 (fp32) or 2 (bf16) bytes per element and does one compare
 // per element, so it is bound by HBM.  Same buffer plans and tiling scheme as
 // the digest kernel (apc_digest.cu), with its own shape: 16-byte aligned
-// bodies in tiles of kCountTile elements over a persistent grid, loads issued for the whole
-// tile before counting, scalar head and tail by the CTA that owns the first
-// tile, per-slot running counts flushed on CTA-uniform slot changes.
+// bodies in tiles of kCountTile elements over a persistent grid, loads
+// issued for the whole tile before counting, scalar head and tail by the CTA
+// that owns the first tile, per-slot running counts flushed on CTA-uniform
+// slot changes.
 #include <cuda_runtime.h>
 
 #include "../../include/apc.h"
