@@ -18,7 +18,7 @@
 //    and, for each, waits until a ring stage is free and issues four
 //    bulk asynchronous copies -- p, m, v and g -- that complete on the
 //    stage's "full" mbarrier.  Loads never occupy consumer registers, and up
-//    to kCommitStages tiles per CTA are in flight.
+//    to L::kStages tiles per CTA are in flight.
 //  * With each stage the producer also writes a 48-byte descriptor (the
 //    tile's first-element addresses in p, m, v, w, g, its element count and
 //    first digest index) into shared memory before arming the stage, so the
@@ -127,6 +127,7 @@ struct F32State {
   static constexpr uint32_t kES = 4;        // bytes per state element
   static constexpr int kDigests = 4;
   static constexpr int kConsumerWarps = kCommitConsumerWarps;
+  static constexpr int kStages = kCommitStages;
   static constexpr int kConsumers = 32 * kConsumerWarps;
   static constexpr int kThreads = kConsumers + 32;  // + the producer warp
   static constexpr int kBoundThreads = kThreads > APC_COMMIT_BOUND_THREADS ? kThreads : APC_COMMIT_BOUND_THREADS;
@@ -212,6 +213,7 @@ struct BF16State {
   static constexpr uint32_t kES = 2;
   static constexpr int kDigests = 3;
   static constexpr int kConsumerWarps = kCommitConsumerWarpsBF16;
+  static constexpr int kStages = kCommitStagesBF16;
   static constexpr int kConsumers = 32 * kConsumerWarps;
   static constexpr int kThreads = kConsumers + 32;
   static constexpr int kBoundThreads = kThreads;
@@ -323,7 +325,7 @@ __host__ __device__ constexpr uint32_t stage_bytes() {
 
 template <class L>
 __host__ __device__ constexpr uint32_t smem_bytes() {
-  return (uint32_t)kCommitStages * stage_bytes<L>();
+  return (uint32_t)L::kStages * stage_bytes<L>();
 }
 
 static_assert(smem_bytes<F32State>() <= 227 * 1024 && smem_bytes<BF16State>() <= 227 * 1024, "shared memory per CTA");
@@ -353,15 +355,15 @@ template <class L, int MAXE, bool ZERO>
 __global__ void __launch_bounds__(L::kBoundThreads, kCommitBlocksPerSm)
     commit_kernel(const __grid_constant__ CommitPlan<MAXE> plan, unsigned long long *out) {
   extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ __align__(8) uint64_t full[kCommitStages];
-  __shared__ __align__(8) uint64_t empty[kCommitStages];
-  __shared__ StageDesc desc[kCommitStages];
+  __shared__ __align__(8) uint64_t full[L::kStages];
+  __shared__ __align__(8) uint64_t empty[L::kStages];
+  __shared__ StageDesc desc[L::kStages];
   __shared__ uint64_t red[L::kThreads / 32];
   __shared__ int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kCommitStages; ++s) {
+    for (int s = 0; s < L::kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], L::kConsumerWarps);
     }
@@ -406,17 +408,17 @@ __global__ void __launch_bounds__(L::kBoundThreads, kCommitBlocksPerSm)
                  cnt * L::kES, &full[stage], policy);
         bulk_g2s(st + 3 * L::kES * L::kTile, E.g + start, cnt * 2, &full[stage], policy);
         ++issued;
-        if (++stage == kCommitStages) {
+        if (++stage == L::kStages) {
           stage = 0;
           phase ^= 1;
         }
       }
       // Drain: the last min(issued, stages) copies must have landed before
       // the CTA may exit (normally the consumers already waited for them).
-      const int n_drain = (int)umin64(issued, (uint64_t)kCommitStages);
+      const int n_drain = (int)umin64(issued, (uint64_t)L::kStages);
       for (int k = 0; k < n_drain; ++k) {
         if (--stage < 0) {
-          stage = kCommitStages - 1;
+          stage = L::kStages - 1;
           phase ^= 1;
         }
         if (!mbar_wait(&full[stage], phase)) atomicOr(&g_commit_status, (unsigned)APC_ETIMEOUT);
@@ -453,7 +455,7 @@ __global__ void __launch_bounds__(L::kBoundThreads, kCommitBlocksPerSm)
       const Dst d{sd.p + ob * L::kES, sd.m + ob * L::kES, sd.v + ob * L::kES,
                   L::kDigests == 4 ? sd.w + ob : nullptr, sd.g + ob};
       store_groups<L, ZERO, 0>(d, sd.G + ob, r, ok, s, a);
-      if (++stage == kCommitStages) {
+      if (++stage == L::kStages) {
         stage = 0;
         phase ^= 1;
       }
